@@ -1,0 +1,207 @@
+/*
+ * viscache.h -- C ABI of libviscache, the GB300 (sm_103a) PruneKV visual-KV
+ * compression pass of VisCache (Sec. 3.2 and Algorithm 1 of the paper).
+ *
+ * The pass runs once per request after prefill.  Per request it
+ *   (a) scores every visual token by the attention the observation-window
+ *       query rows pay it, summed over query heads and layers   -- Eq. (token_score);
+ *   (b) keeps the top-B_l tokens of each KV head in layer l, B_l from the
+ *       parabolic schedule, and evicts layers l > h            -- Eq. (parabolic);
+ *   (c) drops the keys of the other survivors and fuses their values into
+ *       the kept values                                         -- Eq. (redistribution),
+ *                                                                  Eq. (weight_fusion);
+ *   (d) writes the result as a dense variable-length cache.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every function returns an int status (VC_OK = 0 or a VC_ERR_* code).
+ *   Nothing is printed; no C++ exception crosses the ABI.
+ * - The caller owns every buffer.  The library never allocates device
+ *   memory: scratch space comes from a caller workspace ("ws") whose size the
+ *   matching *_workspace_size function returns.  ws must be 256-byte aligned.
+ * - Device work is queued on the caller's stream (a cudaStream_t passed as
+ *   void*, NULL = legacy default stream) and is asynchronous; after a stream
+ *   synchronisation prunekv_get_status(ws) reports device-side errors
+ *   (a bounded wait that timed out, an index out of range).
+ * - Tensors are dense, row-major, passed as device pointers, element type
+ *   VC_BF16 (bfloat16) or VC_F32 (float32); data pointers must be 16-byte
+ *   aligned.  Layouts, per request (GQA: query head j reads KV head j / G,
+ *   G = Hq / Hkv):
+ *       Qw [L][Hq][W][d]    observation-window query rows (the last W rows)
+ *       K  [L][Hkv][n][d]   visual keys   (n = n_vis)
+ *       V  [L][Hkv][n][d]   visual values
+ * - Compressed output ("dense varlen", D8): with P_l = sum_{j<l} B_j, layer l
+ *   of a request is a [Hkv][B_l][d] block starting at row Hkv * P_l; the kept
+ *   positions idx[Hkv][B_l] sit at the same row offsets.  Rows are in
+ *   ascending original position.  Layers l > h (B_l = 0) are absent.
+ *   Drop lists use the same scheme with D_l = Nq - B_l (l <= h, B_l > 0).
+ * - Supported: d in {64, 128}; 1 <= n <= 65536; W >= 1; Hq % Hkv == 0;
+ *   L <= 256.  The library is stateless and thread-safe.
+ */
+#ifndef VISCACHE_H_
+#define VISCACHE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---- */
+#define VC_OK                   0
+#define VC_ERR_INVALID_ARG      1  /* bad size, mode, pointer alignment, mu/tau range */
+#define VC_ERR_INFEASIBLE       2  /* retention target cannot be met (B_1 > n) */
+#define VC_ERR_WORKSPACE        3  /* workspace NULL, misaligned or smaller than required */
+#define VC_ERR_CUDA             4  /* a CUDA runtime call or kernel launch failed */
+#define VC_ERR_DEVICE_TIMEOUT   5  /* a bounded device-side wait gave up */
+#define VC_ERR_UNSUPPORTED      6  /* valid request outside what this build implements */
+#define VC_ERR_DEVICE_INDEX     7  /* a kernel met an index out of range and skipped it */
+
+/* ---- element types ---- */
+#define VC_BF16 0
+#define VC_F32  1
+
+/* ---- ranking modes (Sec. 4.4: shared global vs. layer-specific ranking) ---- */
+#define VC_RANK_SHARED    0  /* one order per KV head from the 1/L layer mean (default) */
+#define VC_RANK_PER_LAYER 1  /* one order per (layer, KV head) */
+
+/*
+ * viscache_plan_budgets -- parabolic layer budgets, host only, exact integers.
+ *
+ * Paper: Eq. (parabolic) b_l = 1 - (l-1)^2 / (2 (h-1)^2) for l <= h, layers
+ * l > h evicted, normalised to sum_l b_l = h*m; RR = p*q*(h/L)*m (Sec. 4,
+ * Implementation Details) with p = 1.
+ * Reading: T = round(RR * n * L) kept (token, layer) pairs per KV head,
+ * split over layers 1..h in proportion to b_l by largest remainder (ties to
+ * the lower layer); survivors Nq = round(T / (h*m)), at least B_1, at most n.
+ * round() is round-half-up on exact rationals.
+ *
+ *   L, n_vis        layers, visual tokens (>= 1)
+ *   rr_num/rr_den   overall retention RR in (0, 1]
+ *   h               truncation layer in [1, L]; 0 selects round(3L/4)
+ *                   clamped to [min(2, L), L]
+ *   m_num/m_den     average layer budget m in (0, 1]; m_den = 0 selects 3/4
+ *   B_out           host int32[L]: B_l (0 for l > h), non-increasing
+ *   n_survive_out   host int32: Nq
+ *   h_out           host int32 (nullable): the truncation layer used
+ * Errors: VC_ERR_INVALID_ARG (ranges, NULL outputs), VC_ERR_INFEASIBLE (B_1 > n).
+ */
+int viscache_plan_budgets(int32_t L, int32_t n_vis, uint32_t rr_num, uint32_t rr_den,
+                          int32_t h, uint32_t m_num, uint32_t m_den,
+                          int32_t* B_out, int32_t* n_survive_out, int32_t* h_out);
+
+/*
+ * prunekv_score -- token importance, Eq. (token_score) / Algorithm 1 step 1.
+ *
+ *   s[g][v]    = (1/L) sum_l sum_{j in group g} sum_i A^l_{j,i,v}   (VC_RANK_SHARED)
+ *   s[l][g][v] =       sum_{j in group g} sum_i A^l_{j,i,v}         (VC_RANK_PER_LAYER)
+ *   A^l_{j,i,v} = softmax over the n visual keys of scale * q^l_{j,i} . k^l_{j/G,v}
+ *
+ * With row_lse (device float[L][Hq][W], natural log, nullable) the
+ * normaliser is taken from the caller instead: A = exp(scale*q.k - lse).
+ *   Qw, K       device, dtype, layouts above
+ *   scale       0 selects 1/sqrt(d)
+ *   scores      device float32 output, [Hkv][n] or [L][Hkv][n]
+ *   ws          workspace of prunekv_score_workspace_size(L, Hq, W) bytes
+ * Arithmetic: bf16 inputs are multiplied exactly and accumulated in fp32;
+ * softmax and sums in fp32.
+ */
+size_t prunekv_score_workspace_size(int32_t L, int32_t Hq, int32_t W);
+int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq,
+                  int32_t Hkv, int32_t d, int32_t n_vis, int32_t W, float scale,
+                  int rank_mode, const float* row_lse, float* scores,
+                  void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * prunekv_select -- rank, keep and drop sets, Algorithm 1 steps 1 and 3.
+ *
+ * Per KV head (per (layer, KV head) in VC_RANK_PER_LAYER) tokens are ordered
+ * by descending score, the lower index first on exact ties.  The first Nq are
+ * the survivors ("retain the q percent", the rest discarded); layer l keeps
+ * the first B_l and drops survivors B_l .. Nq-1.
+ *   scores      device float32 from prunekv_score
+ *   B           HOST int32[L] budgets (from viscache_plan_budgets), B_l <= Nq <= n
+ *   rank_out    device int32 [Hkv][n] (or [L][Hkv][n]): position of each token
+ *   keep_idx    device int32, rows Hkv*P_l + g*B_l + r: kept positions, ascending
+ *   drop_idx    device int32, rows Hkv*Q_l + g*D_l + r, D_l = Nq - B_l,
+ *               Q_l = sum_{j<l, B_j>0} D_j: dropped survivors, ascending
+ *   ws          workspace of prunekv_select_workspace_size(...) bytes
+ */
+size_t prunekv_select_workspace_size(int32_t L, int32_t Hkv, int32_t n_vis, int rank_mode);
+int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis,
+                   const int32_t* B, int32_t Nq, int rank_mode, int32_t* rank_out,
+                   int32_t* keep_idx, int32_t* drop_idx, void* ws, size_t ws_bytes,
+                   void* stream);
+
+/*
+ * prunekv_fuse_compact -- prune keys, fuse values, compact; Algorithm 1 step 3.
+ *
+ *   K_out = K[keep]                                  (bit-exact copy)
+ *   V_out = mu * V_k + (1 - mu) * Phi V_d,  Phi = row-softmax(V_k V_d^T / tau)
+ *           -- Eq. (redistribution), Eq. (weight_fusion); V_out = V_k when the
+ *           drop set is empty.  fp32 arithmetic, rounded to dtype (RNE).
+ *   K, V              device [L][Hkv][n][d], dtype
+ *   B, Nq             HOST budgets as for prunekv_select
+ *   keep_idx/drop_idx device lists from prunekv_select
+ *   mu in [0, 1], tau > 0
+ *   K_out, V_out      device, dense varlen (rows Hkv * sum_l B_l, d columns)
+ *   ws                workspace of prunekv_fuse_workspace_size(L) bytes
+ */
+size_t prunekv_fuse_workspace_size(int32_t L);
+int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int32_t Hkv,
+                         int32_t d, int32_t n_vis, const int32_t* B, int32_t Nq,
+                         const int32_t* keep_idx, const int32_t* drop_idx, float mu,
+                         float tau, void* K_out, void* V_out, void* ws, size_t ws_bytes,
+                         void* stream);
+
+/*
+ * prunekv_compress -- the whole pass for a batch of requests in one call:
+ * plan (host), score, select, fuse and compact, queued on one stream.
+ *
+ * Requests share the model shape (L, Hq, Hkv, d) and differ in n, W and RR.
+ * Inputs are packed request after request, each request laid out exactly as
+ * a single request:  K/V of request r start at element L*Hkv*d*sum_{r'<r} n_r',
+ * Qw of request r at element L*Hq*d*sum_{r'<r} W_r'.  Outputs likewise: request
+ * r's dense varlen cache starts at row Hkv * sum_{r'<r} T_r' (T_r = sum_l B_l).
+ */
+typedef struct {
+    int32_t n_req;            /* number of requests, >= 1 */
+    const int32_t* n_vis;     /* host [n_req] visual tokens per request */
+    const int32_t* W;         /* host [n_req] window rows per request */
+    const uint32_t* rr_num;   /* host [n_req] retention numerators */
+    const uint32_t* rr_den;   /* host [n_req] retention denominators */
+} vc_batch;
+
+typedef struct {
+    int32_t L, Hq, Hkv, d;    /* model shape */
+    int32_t dtype;            /* VC_BF16 or VC_F32 */
+    int32_t h;                /* truncation layer, 0 = round(3L/4) */
+    uint32_t m_num, m_den;    /* average layer budget m, m_den = 0 -> 3/4 */
+    float mu;                 /* fusion strength, paper default 0.7 */
+    float tau;                /* redistribution temperature, paper default 1.0 */
+    float scale;              /* logit scale, 0 -> 1/sqrt(d) */
+    int32_t rank_mode;        /* VC_RANK_SHARED or VC_RANK_PER_LAYER */
+} vc_params;
+
+size_t prunekv_workspace_size(const vc_batch* batch, const vc_params* p);
+int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw,
+                     const void* K, const void* V, void* K_out, void* V_out,
+                     int32_t* idx_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * prunekv_get_status -- device-side status of the last call that used ws.
+ * Synchronises the stream, returns VC_OK or the first device error code
+ * recorded (VC_ERR_DEVICE_TIMEOUT, VC_ERR_DEVICE_INDEX), or VC_ERR_CUDA.
+ * Every entry point clears the status word when it starts.
+ */
+int prunekv_get_status(const void* ws, void* stream);
+
+/* Version string of the library build. */
+const char* viscache_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VISCACHE_H_ */

@@ -1,0 +1,415 @@
+#!/usr/bin/env python
+"""Throughput of the PruneKV visual-KV compression pass on GB300.
+
+One step = one prunekv_compress call (plan, score, select, fuse, compact) over
+one request of the selected workload (default: 7B shape, 28 layers, 28/4
+heads, d=128, 64 frames x 196 = 12,544 visual tokens, 64 window rows, 19%
+retention, bf16).  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 3] [--impl ours|reference]
+
+--impl reference times the fp64 CPU oracle (the slow, obviously correct
+program the CUDA path is checked against) on bounded samples of the same
+workload, on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "PruneKV visual-KV tokens×layers compressed/s at 1 GB300; % of roofline"
+UNIT = "tokens*layers/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=p["hbm_gbs"], tc=p["bf16_tflops"], tc_sus=p.get("bf16_tflops_sustained"),
+                    source="measured")
+    return dict(hbm=6800.0, tc=1900.0, tc_sus=1700.0, source="fallback")
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic work of one pass (what the method must do, each logit once).
+
+def plans_for(wl, vc):
+    out = []
+    for r in wl.requests:
+        B, Nq, h = vc.viscache_plan_budgets(wl.L, r.n, r.rr_num, r.rr_den)
+        out.append((B, Nq, h))
+    return out
+
+
+def algorithmic(wl, plans):
+    eb = 2 if wl.dtype == "bf16" else 4
+    tot = dict(bytes=0, flops_score=0, flops_fuse=0, k_bytes=0, gather_bytes=0, fuse_bytes=0,
+               tokens_layers=0)
+    for r, (B, Nq, h) in zip(wl.requests, plans):
+        T = sum(B)
+        row = wl.d * eb
+        k_all = wl.L * wl.Hkv * r.n * row
+        q = wl.L * wl.Hq * r.W * row
+        kept_k = wl.Hkv * T * row
+        surv_v = sum(1 for b in B if b > 0) * wl.Hkv * Nq * row
+        out = 2 * wl.Hkv * T * row
+        tot["bytes"] += k_all + q + kept_k + surv_v + out
+        tot["k_bytes"] += k_all + q
+        tot["gather_bytes"] += 2 * kept_k
+        tot["fuse_bytes"] += surv_v + wl.Hkv * T * row
+        tot["flops_score"] += 2 * wl.Hq * r.W * r.n * wl.d * wl.L
+        tot["flops_fuse"] += 4 * wl.Hkv * wl.d * sum(b * (Nq - b) for b in B if b > 0)
+        tot["tokens_layers"] += r.n * wl.L
+    return tot
+
+
+# per kernel: (kind, work key) -> achieved = work / time
+KERNEL_WORK = {
+    "score_lse_simt": ("tensor", "flops_score"),
+    "score_colsum_simt": ("tensor", "flops_score"),
+    "score_lse_tc": ("tensor", "flops_score"),
+    "score_colsum_tc": ("tensor", "flops_score"),
+    "fuse_v_simt": ("tensor", "flops_fuse"),
+    "fuse_v_tc": ("tensor", "flops_fuse"),
+    "gather_k": ("hbm", "gather_bytes"),
+}
+
+
+def traffic_for(kernel):
+    """dram bytes per launch from a committed ncu summary, if the kernel source is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        tab = json.load(f)
+    ent = tab.get(kernel)
+    if not ent:
+        return None
+    src = os.path.join(ROOT, ent["source"])
+    if not os.path.exists(src):
+        return None
+    with open(src, "rb") as f:
+        digest = hashlib.sha256(f.read()).hexdigest()[:16]
+    return ent["dram_bytes_per_launch"] if digest == ent["source_sha256_16"] else None
+
+
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "200", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, layers, seed_layer0=0):
+    """Run the fp64 oracle on the first `layers` layers of request 0; returns (seconds, tokens*layers)."""
+    import numpy as np
+    import torch
+    from fractions import Fraction
+
+    from oracle import plan as oplan
+    from oracle import prunekv as ok
+    from paper_2608_24063_gb300 import synth
+
+    sub = synth.scaled(wl, "sample", L=layers, requests=[wl.requests[0]])
+    q = synth.make_q(sub, 0)
+    k, v = synth.make_kv(sub, 0, q)
+    Qn, Kn, Vn = (t.to(torch.float64).numpy() for t in (q, k, v))
+    r = sub.requests[0]
+    B, Nq, h = oplan.plan_budgets(layers, r.n, Fraction(r.rr_num, r.rr_den))
+    t0 = time.perf_counter()
+    ok.prunekv(Qn, Kn, Vn, B, Nq, mu=0.7, tau=1.0)
+    dt = time.perf_counter() - t0
+    return dt, r.n * layers
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args, wl):
+    """--impl reference: the oracle timed on the host cores, one bounded sample per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    layers = 1
+    for _ in range(args.warmup):
+        oracle_sample(wl, layers)
+    times = []
+    tl = 0
+    for _ in range(args.steps):
+        dt, tl = oracle_sample(wl, layers)
+        times.append(dt)
+    sec = sum(times) / len(times)
+    val = tl / sec
+    cfg = workload_config(wl)
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded, structure of the paper's long-video workloads)",
+            "config": cfg,
+            "cpu_baseline": {"value": val, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                             "sample": "Algorithm 1 on layer 1 of %d (all %d tokens, %d window rows) per step" %
+                                       (wl.L, wl.requests[0].n, wl.requests[0].W)},
+            "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(wl):
+    r = wl.requests[0]
+    in_bytes = sum(wl.L * (wl.Hq * q.W + 2 * wl.Hkv * q.n) * wl.d * (2 if wl.dtype == "bf16" else 4)
+                   for q in wl.requests)
+    return {"workload": wl.name, "requests": len(wl.requests), "L": wl.L, "Hq": wl.Hq,
+            "Hkv": wl.Hkv, "d": wl.d, "n_vis": [q.n for q in wl.requests],
+            "W": [q.W for q in wl.requests],
+            "retention": ["%d/%d" % (q.rr_num, q.rr_den) for q in wl.requests],
+            "h": "3L/4", "m": 0.75, "mu": 0.7, "tau": 1.0, "rank": "shared",
+            "l2": "inputs larger than L2 (%.2f GB of Qw+K+V > 129 MB)" % (in_bytes / 1e9)}
+
+
+def main():
+    args = parse()
+    from paper_2608_24063_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_24063_gb300 import viscache as vc
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    st = torch.cuda.current_stream()
+
+    # inputs: generated on the device, resident in HBM before timing
+    qs, ks, vs = synth.generate(wl, dev)
+    Q = torch.cat([q.flatten() for q in qs]) if len(qs) > 1 else qs[0]
+    K = torch.cat([k.flatten() for k in ks]) if len(ks) > 1 else ks[0]
+    V = torch.cat([v.flatten() for v in vs]) if len(vs) > 1 else vs[0]
+    del qs, ks, vs
+    batch = vc.Batch([r.n for r in wl.requests], [r.W for r in wl.requests],
+                     [(r.rr_num, r.rr_den) for r in wl.requests])
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16 if wl.dtype == "bf16" else vc.VC_F32)
+    rows = vc.compressed_rows(batch, prm)
+    K_out = torch.empty((rows, wl.d), dtype=K.dtype, device=dev)
+    V_out = torch.empty((rows, wl.d), dtype=V.dtype, device=dev)
+    idx = torch.empty(rows, dtype=torch.int32, device=dev)
+    ws = torch.empty(vc.prunekv_workspace_size(batch, prm), dtype=torch.uint8, device=dev)
+
+    def step():
+        vc.prunekv_compress(batch, prm, Q, K, V, K_out, V_out, idx, ws)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    vc.viscache_profile_enable(True)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(st)
+    for _ in range(args.steps):
+        step()
+    t1.record(st)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    kern = vc.viscache_profile_read()
+    vc.viscache_profile_enable(False)
+    clk = clocks.stop()
+    ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / args.steps
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+
+    plans = plans_for(wl, vc)
+    work = algorithmic(wl, plans)
+    value = world * work["tokens_layers"] / (ms_step * 1e-3)
+    pk = peaks()
+
+    # dominant kernel
+    dom = max(kern.items(), key=lambda kv: kv[1][0]) if kern else None
+    roof = None
+    if dom:
+        name, (tot_ms, launches) = dom
+        kind, key = KERNEL_WORK.get(name, ("hbm", "bytes"))
+        per = tot_ms / max(launches, 1) * 1e-3
+        if kind == "tensor":
+            ach = work[key] / per / 1e12
+            roof = {"kernel": name, "bound": "tensor", "achieved": ach, "peak": pk["tc"],
+                    "unit": "TFLOP/s", "frac": ach / pk["tc"], "traffic": traffic_for(name),
+                    "peak_source": pk["source"] + " bf16 dense burst"}
+        else:
+            ach = work[key] / per / 1e9
+            roof = {"kernel": name, "bound": "hbm", "achieved": ach, "peak": pk["hbm"],
+                    "unit": "GB/s", "frac": ach / pk["hbm"], "traffic": traffic_for(name),
+                    "peak_source": pk["source"] + " copy bandwidth"}
+    t_hbm = work["bytes"] / (pk["hbm"] * 1e9)
+    t_tc = work["flops_score"] / (pk["tc"] * 1e12)
+    t_fuse = work["flops_fuse"] / (pk["tc"] * 1e12)
+    pass_roof = {"t_roofline_us": max(t_hbm, t_tc) * 1e6, "frac": max(t_hbm, t_tc) / (ms_step * 1e-3),
+                 "t_roofline_incl_fusion_us": max(t_hbm, t_tc + t_fuse) * 1e6,
+                 "frac_incl_fusion": max(t_hbm, t_tc + t_fuse) / (ms_step * 1e-3),
+                 "bytes": work["bytes"], "flops_score": work["flops_score"],
+                 "flops_fuse": work["flops_fuse"]}
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        hQ = torch.empty(Q.shape, dtype=Q.dtype, pin_memory=True)
+        hK = torch.empty(K.shape, dtype=K.dtype, pin_memory=True)
+        hV = torch.empty(V.shape, dtype=V.dtype, pin_memory=True)
+        hQ.copy_(Q); hK.copy_(K); hV.copy_(V)
+        oK = torch.empty(K_out.shape, dtype=K_out.dtype, pin_memory=True)
+        oV = torch.empty(V_out.shape, dtype=V_out.dtype, pin_memory=True)
+        oI = torch.empty(idx.shape, dtype=idx.dtype, pin_memory=True)
+        dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+
+        def e2e_step():
+            dQ.copy_(hQ, non_blocking=True)
+            dK.copy_(hK, non_blocking=True)
+            dV.copy_(hV, non_blocking=True)
+            vc.prunekv_compress(batch, prm, dQ, dK, dV, K_out, V_out, idx, ws)
+            oK.copy_(K_out, non_blocking=True)
+            oV.copy_(V_out, non_blocking=True)
+            oI.copy_(idx, non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        torch.cuda.synchronize()
+        e_steps = max(3, min(args.steps, 10))
+        if world > 1:
+            dist.barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(st)
+        for _ in range(e_steps):
+            e2e_step()
+        b.record(st)
+        torch.cuda.synchronize()
+        ems = a.elapsed_time(b) / e_steps
+        if world > 1:
+            tt = torch.tensor([ems], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ems = float(tt.item())
+        e2e = {"value": world * work["tokens_layers"] / (ems * 1e-3), "unit": UNIT,
+               "ms_per_step": ems,
+               "h2d_bytes_per_step": int(Q.numel() * Q.element_size() + K.numel() * K.element_size()
+                                         + V.numel() * V.element_size()),
+               "d2h_bytes_per_step": int(K_out.numel() * K_out.element_size()
+                                         + V_out.numel() * V_out.element_size()
+                                         + idx.numel() * idx.element_size())}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        dt1, tl1 = oracle_sample(wl, 1)
+        layers = max(1, min(wl.L, int(args.cpu_seconds / max(dt1, 1e-3))))
+        dt, tl = oracle_sample(wl, layers) if layers > 1 else (dt1, tl1)
+        cpu = {"value": tl / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": "Algorithm 1 (fp64 numpy) on the first %d of %d layers of the workload's "
+                         "request (all %d tokens, %d window rows): %.1f s" %
+                         (layers, wl.L, wl.requests[0].n, wl.requests[0].W, dt)}
+
+    launches = sum(c for _, c in kern.values())
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16"
+                if wl.dtype == "bf16" else "f32",
+                "data": "synthetic (seeded, structure of the paper's long-video workloads)",
+                "config": workload_config(wl), "roofline": roof, "pass_roofline": pass_roof,
+                "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "kernels_ms_per_step": {k: v[0] / args.steps for k, v in kern.items()},
+                "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -197,6 +197,19 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw,
  */
 int prunekv_get_status(const void* ws, void* stream);
 
+/*
+ * Benchmark support (not a step of the pass): per-kernel CUDA-event timing.
+ * viscache_profile_enable(1) makes every later kernel launch record an event
+ * pair on its stream (and clears what was recorded); viscache_profile_read
+ * waits for the recorded events, writes up to max_kernels entries -- kernel
+ * names joined by '\n' into names (name_bytes long), summed milliseconds and
+ * launch counts -- clears the record and returns the number of entries, or
+ * -VC_ERR_CUDA if an event could not be read.  Not thread-safe; off by default.
+ */
+int viscache_profile_enable(int on);
+int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* launches,
+                          int max_kernels);
+
 /* Version string of the library build. */
 const char* viscache_version(void);
 

@@ -1,0 +1,403 @@
+// C ABI of libviscache (declared in include/viscache.h): argument checks,
+// workspace layout, device plan tables and kernel launches.  Every step of
+// the pass runs in this library's kernels; nothing here computes on the host
+// except the integer budget plan and the table offsets.
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <vector>
+
+#include "kernels.h"
+#include "vc_common.cuh"
+
+namespace vc {
+namespace {
+
+constexpr size_t kAlign = 256;
+inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Sequential carving of the caller workspace into 256-byte aligned regions.
+struct Arena {
+  size_t off = 0;
+  size_t take(size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes);
+    return o;
+  }
+};
+
+struct RequestPlan {
+  int32_t n = 0, W = 0, Nq = 0, h = 0;
+  std::vector<int32_t> B;
+};
+
+// Host image of the device tables plus the workspace offsets of every region.
+struct Layout {
+  // inputs
+  int n_req = 0, L = 0, Hq = 0, Hkv = 0, d = 0, rank_mode = VC_RANK_SHARED;
+  bool need_lse = false, need_scores = false, need_sort = false, need_drop = false;
+  // derived sizes
+  int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
+  int units_lse = 0, units_col = 0, units_fuse = 0;
+  // workspace offsets
+  size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
+         o_row0 = 0, table_begin = 0, table_end = 0, o_lse = 0, o_scores = 0, o_keys = 0,
+         o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
+  // host images
+  std::vector<Req> req;
+  std::vector<Layer> layer;
+  std::vector<int32_t> u_lse, u_col, u_fuse;
+  std::vector<int64_t> row0;
+
+  void build(const std::vector<RequestPlan>& plans) {
+    n_req = (int)plans.size();
+    const int G = Hq > 0 && Hkv > 0 ? Hq / Hkv : 1;
+    req.assign(n_req, Req{});
+    layer.assign((size_t)n_req * L, Layer{});
+    u_lse.assign(n_req + 1, 0);
+    u_col.assign(n_req + 1, 0);
+    u_fuse.assign((size_t)n_req * L + 1, 0);
+    row0.assign((size_t)n_req * L + 1, 0);
+    int64_t cu_n = 0, cu_w = 0;
+    const int per_req_problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
+    const int rows_tile = score_rows_per_tile_simt(), keys_tile = score_keys_per_tile_simt();
+    const int fuse_tile = fuse_rows_per_tile_simt();
+    for (int r = 0; r < n_req; ++r) {
+      const RequestPlan& p = plans[r];
+      Req& q = req[r];
+      q.kv_off = (int64_t)L * Hkv * d * cu_n;
+      q.q_off = (int64_t)L * Hq * d * cu_w;
+      q.lse_off = (int64_t)L * Hq * cu_w;
+      q.s_off = (int64_t)per_req_problems * cu_n;
+      q.out_row0 = out_rows;
+      q.drop_row0 = drop_rows;
+      q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
+      u_lse[r + 1] = u_lse[r] + (G * p.W + rows_tile - 1) / rows_tile;
+      u_col[r + 1] = u_col[r] + (p.n + keys_tile - 1) / keys_tile;
+      int32_t P = 0, Qd = 0;
+      for (int l = 0; l < L; ++l) {
+        const size_t rl = (size_t)r * L + l;
+        const int32_t b = p.B.empty() ? 0 : p.B[l];
+        Layer& ly = layer[rl];
+        ly.B = b; ly.P = P; ly.D = b > 0 ? p.Nq - b : 0; ly.Qd = Qd;
+        row0[rl] = out_rows + (int64_t)Hkv * P;
+        u_fuse[rl + 1] = u_fuse[rl] + Hkv * ((b + fuse_tile - 1) / fuse_tile);
+        P += b;
+        Qd += ly.D;
+      }
+      out_rows += (int64_t)Hkv * P;
+      drop_rows += (int64_t)Hkv * Qd;
+      cu_n += p.n;
+      cu_w += p.W;
+    }
+    row0[(size_t)n_req * L] = out_rows;
+    lse_elems = (int64_t)L * Hq * cu_w;
+    score_elems = (int64_t)per_req_problems * cu_n;
+    units_lse = u_lse[n_req];
+    units_col = u_col[n_req];
+    units_fuse = u_fuse[(size_t)n_req * L];
+
+    Arena a;
+    o_status = a.take(kAlign);
+    table_begin = a.off;
+    o_req = a.take(sizeof(Req) * n_req);
+    o_layer = a.take(sizeof(Layer) * layer.size());
+    o_u_lse = a.take(sizeof(int32_t) * u_lse.size());
+    o_u_col = a.take(sizeof(int32_t) * u_col.size());
+    o_u_fuse = a.take(sizeof(int32_t) * u_fuse.size());
+    o_row0 = a.take(sizeof(int64_t) * row0.size());
+    table_end = a.off;
+    if (need_lse) o_lse = a.take(sizeof(float) * lse_elems);
+    if (need_scores) o_scores = a.take(sizeof(float) * score_elems);
+    if (need_sort) {
+      o_keys = a.take(sizeof(uint32_t) * 2 * score_elems);
+      o_vals = a.take(sizeof(int32_t) * 2 * score_elems);
+      if (need_scores) o_rank = a.take(sizeof(int32_t) * score_elems);
+    }
+    if (need_drop) o_drop = a.take(sizeof(int32_t) * drop_rows);
+    total = a.off;
+  }
+
+  // Copy the table image into the workspace and clear the status word.  Small
+  // images (every single request and typical batches) travel as a kernel
+  // parameter, so the upload is an ordinary launch on the stream (no host
+  // blocking, capturable in a CUDA graph); larger ones use one memcpy.
+  cudaError_t upload(uint8_t* ws, cudaStream_t st) const {
+    const size_t bytes = table_end - table_begin;
+    if (bytes <= sizeof(TableImage::bytes)) {
+      TableImage im;
+      memset(&im, 0, sizeof(im));
+      fill(im.bytes);
+      return launch_upload(im, (uint32_t)bytes, ws + table_begin,
+                           reinterpret_cast<int32_t*>(ws + o_status), st);
+    }
+    std::vector<uint8_t> img(bytes, 0);
+    fill(img.data());
+    cudaError_t e = cudaMemsetAsync(ws + o_status, 0, kAlign, st);
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyAsync(ws + table_begin, img.data(), bytes, cudaMemcpyHostToDevice, st);
+  }
+
+  void fill(uint8_t* img) const {
+    auto put = [&](size_t off, const void* src, size_t n) {
+      if (n) memcpy(img + (off - table_begin), src, n);
+    };
+    put(o_req, req.data(), sizeof(Req) * req.size());
+    put(o_layer, layer.data(), sizeof(Layer) * layer.size());
+    put(o_u_lse, u_lse.data(), sizeof(int32_t) * u_lse.size());
+    put(o_u_col, u_col.data(), sizeof(int32_t) * u_col.size());
+    put(o_u_fuse, u_fuse.data(), sizeof(int32_t) * u_fuse.size());
+    put(o_row0, row0.data(), sizeof(int64_t) * row0.size());
+  }
+
+  Tables tables(uint8_t* ws) const {
+    Tables t;
+    t.req = reinterpret_cast<const Req*>(ws + o_req);
+    t.layer = reinterpret_cast<const Layer*>(ws + o_layer);
+    t.unit0_lse = reinterpret_cast<const int32_t*>(ws + o_u_lse);
+    t.unit0_col = reinterpret_cast<const int32_t*>(ws + o_u_col);
+    t.unit0_fuse = reinterpret_cast<const int32_t*>(ws + o_u_fuse);
+    t.row0_out = reinterpret_cast<const int64_t*>(ws + o_row0);
+    t.status = reinterpret_cast<int32_t*>(ws + o_status);
+    return t;
+  }
+
+  Shape shape(float scale) const {
+    Shape s;
+    s.L = L; s.Hq = Hq; s.Hkv = Hkv; s.d = d; s.G = (Hq > 0 && Hkv > 0) ? Hq / Hkv : 1;
+    s.n_req = n_req;
+    s.rank_mode = rank_mode;
+    s.scale_log2 = scale * kLog2e;
+    return s;
+  }
+};
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool valid_model(int dtype, int L, int Hq, int Hkv, int d) {
+  if (dtype != VC_BF16 && dtype != VC_F32) return false;
+  if (L < 1 || L > 256 || Hkv < 1 || Hq < Hkv || Hq % Hkv != 0) return false;
+  return d == 64 || d == 128;
+}
+
+int check_ws(const void* ws, size_t ws_bytes, size_t need) {
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return VC_ERR_WORKSPACE;
+  return ws_bytes < need ? VC_ERR_WORKSPACE : VC_OK;
+}
+
+inline int cuda_status(cudaError_t e) { return e == cudaSuccess ? VC_OK : VC_ERR_CUDA; }
+
+// Budgets B (host) must satisfy 0 <= B_l <= Nq <= n.
+bool valid_budgets(const int32_t* B, int L, int Nq, int n) {
+  if (!B || Nq < 0 || Nq > n) return false;
+  for (int l = 0; l < L; ++l)
+    if (B[l] < 0 || B[l] > Nq) return false;
+  return true;
+}
+
+Layout score_layout(int L, int Hq, int Hkv, int d, int n, int W, int rank_mode) {
+  Layout lay;
+  lay.L = L; lay.Hq = Hq; lay.Hkv = Hkv; lay.d = d; lay.rank_mode = rank_mode;
+  lay.need_lse = true;
+  RequestPlan p;
+  p.n = n; p.W = W;
+  lay.build({p});
+  return lay;
+}
+
+Layout select_layout(int L, int Hkv, int n, const int32_t* B, int Nq, int rank_mode) {
+  Layout lay;
+  lay.L = L; lay.Hq = Hkv; lay.Hkv = Hkv; lay.d = 64; lay.rank_mode = rank_mode;
+  lay.need_sort = true;
+  RequestPlan p;
+  p.n = n; p.W = 1; p.Nq = Nq;
+  if (B) p.B.assign(B, B + L);
+  lay.build({p});
+  return lay;
+}
+
+Layout fuse_layout(int L, int Hkv, int d, int n, const int32_t* B, int Nq) {
+  Layout lay;
+  lay.L = L; lay.Hq = Hkv; lay.Hkv = Hkv; lay.d = d;
+  RequestPlan p;
+  p.n = n; p.W = 1; p.Nq = Nq;
+  if (B) p.B.assign(B, B + L);
+  lay.build({p});
+  return lay;
+}
+
+int plan_batch(const vc_batch* b, const vc_params* p, std::vector<RequestPlan>* plans) {
+  if (!b || !p || b->n_req < 1 || !b->n_vis || !b->W || !b->rr_num || !b->rr_den)
+    return VC_ERR_INVALID_ARG;
+  if (!valid_model(p->dtype, p->L, p->Hq, p->Hkv, p->d)) return VC_ERR_INVALID_ARG;
+  if (p->rank_mode != VC_RANK_SHARED && p->rank_mode != VC_RANK_PER_LAYER) return VC_ERR_INVALID_ARG;
+  if (!(p->mu >= 0.f && p->mu <= 1.f) || !(p->tau > 0.f) || !(p->scale >= 0.f))
+    return VC_ERR_INVALID_ARG;
+  plans->assign(b->n_req, RequestPlan{});
+  for (int r = 0; r < b->n_req; ++r) {
+    RequestPlan& q = (*plans)[r];
+    q.n = b->n_vis[r];
+    q.W = b->W[r];
+    if (q.n < 1 || q.n > 65536 || q.W < 1) return VC_ERR_INVALID_ARG;
+    q.B.assign(p->L, 0);
+    const int rc = viscache_plan_budgets(p->L, q.n, b->rr_num[r], b->rr_den[r], p->h, p->m_num,
+                                         p->m_den, q.B.data(), &q.Nq, &q.h);
+    if (rc != VC_OK) return rc;
+  }
+  return VC_OK;
+}
+
+Layout compress_layout(const vc_params* p, const std::vector<RequestPlan>& plans) {
+  Layout lay;
+  lay.L = p->L; lay.Hq = p->Hq; lay.Hkv = p->Hkv; lay.d = p->d; lay.rank_mode = p->rank_mode;
+  lay.need_lse = lay.need_scores = lay.need_sort = lay.need_drop = true;
+  lay.build(plans);
+  return lay;
+}
+
+}  // namespace
+}  // namespace vc
+
+using namespace vc;
+
+extern "C" {
+
+const char* viscache_version(void) { return "viscache-gb300 0.1 (sm_103a)"; }
+
+size_t prunekv_score_workspace_size(int32_t L, int32_t Hq, int32_t W) {
+  if (L < 1 || L > 256 || Hq < 1 || W < 1) return 0;
+  return score_layout(L, Hq, 1, 64, 1, W, VC_RANK_SHARED).total;
+}
+
+int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq, int32_t Hkv,
+                  int32_t d, int32_t n_vis, int32_t W, float scale, int rank_mode,
+                  const float* row_lse, float* scores, void* ws, size_t ws_bytes, void* stream) {
+  if (!valid_model(dtype, L, Hq, Hkv, d) || n_vis < 1 || n_vis > 65536 || W < 1)
+    return VC_ERR_INVALID_ARG;
+  if (rank_mode != VC_RANK_SHARED && rank_mode != VC_RANK_PER_LAYER) return VC_ERR_INVALID_ARG;
+  if (!Qw || !K || !scores || !aligned16(Qw) || !aligned16(K) || !aligned16(scores))
+    return VC_ERR_INVALID_ARG;
+  if (!(scale >= 0.f)) return VC_ERR_INVALID_ARG;
+  if (scale == 0.f) scale = 1.0f / sqrtf((float)d);
+  Layout lay = score_layout(L, Hq, Hkv, d, n_vis, W, rank_mode);
+  const int wc = check_ws(ws, ws_bytes, lay.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = lay.upload(w, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  e = launch_score_simt(dtype, Qw, K, lay.shape(scale), lay.tables(w), lay.units_lse,
+                        lay.units_col, reinterpret_cast<float*>(w + lay.o_lse), row_lse, scores, st);
+  return cuda_status(e);
+}
+
+size_t prunekv_select_workspace_size(int32_t L, int32_t Hkv, int32_t n_vis, int rank_mode) {
+  if (L < 1 || L > 256 || Hkv < 1 || n_vis < 1) return 0;
+  return select_layout(L, Hkv, n_vis, nullptr, 0, rank_mode).total;
+}
+
+int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis, const int32_t* B,
+                   int32_t Nq, int rank_mode, int32_t* rank_out, int32_t* keep_idx,
+                   int32_t* drop_idx, void* ws, size_t ws_bytes, void* stream) {
+  if (L < 1 || L > 256 || Hkv < 1 || n_vis < 1 || n_vis > 65536) return VC_ERR_INVALID_ARG;
+  if (rank_mode != VC_RANK_SHARED && rank_mode != VC_RANK_PER_LAYER) return VC_ERR_INVALID_ARG;
+  if (!scores || !rank_out || !keep_idx || !drop_idx || !valid_budgets(B, L, Nq, n_vis))
+    return VC_ERR_INVALID_ARG;
+  Layout lay = select_layout(L, Hkv, n_vis, B, Nq, rank_mode);
+  const int wc = check_ws(ws, ws_bytes, lay.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = lay.upload(w, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  const int problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
+  e = launch_select(lay.shape(1.f), lay.tables(w), problems, scores, rank_out,
+                    reinterpret_cast<uint32_t*>(w + lay.o_keys),
+                    reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, keep_idx,
+                    drop_idx, st);
+  return cuda_status(e);
+}
+
+size_t prunekv_fuse_workspace_size(int32_t L) {
+  if (L < 1 || L > 256) return 0;
+  return fuse_layout(L, 1, 64, 1, nullptr, 0).total;
+}
+
+int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int32_t Hkv,
+                         int32_t d, int32_t n_vis, const int32_t* B, int32_t Nq,
+                         const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
+                         void* K_out, void* V_out, void* ws, size_t ws_bytes, void* stream) {
+  if (!valid_model(dtype, L, Hkv, Hkv, d) || n_vis < 1 || n_vis > 65536) return VC_ERR_INVALID_ARG;
+  if (!valid_budgets(B, L, Nq, n_vis)) return VC_ERR_INVALID_ARG;
+  if (!(mu >= 0.f && mu <= 1.f) || !(tau > 0.f)) return VC_ERR_INVALID_ARG;
+  if (!K || !V || !keep_idx || !drop_idx || !K_out || !V_out) return VC_ERR_INVALID_ARG;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(K_out) || !aligned16(V_out))
+    return VC_ERR_INVALID_ARG;
+  Layout lay = fuse_layout(L, Hkv, d, n_vis, B, Nq);
+  const int wc = check_ws(ws, ws_bytes, lay.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = lay.upload(w, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  const Shape sh = lay.shape(1.f);
+  const Tables tb = lay.tables(w);
+  e = launch_gather_k(dtype, K, sh, tb, keep_idx, K_out, lay.out_rows, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  e = launch_fuse_simt(dtype, V, sh, tb, keep_idx, drop_idx, mu, tau, V_out, lay.units_fuse, st);
+  return cuda_status(e);
+}
+
+size_t prunekv_workspace_size(const vc_batch* batch, const vc_params* p) {
+  std::vector<RequestPlan> plans;
+  if (plan_batch(batch, p, &plans) != VC_OK) return 0;
+  return compress_layout(p, plans).total;
+}
+
+int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, const void* K,
+                     const void* V, void* K_out, void* V_out, int32_t* idx_out, void* ws,
+                     size_t ws_bytes, void* stream) {
+  std::vector<RequestPlan> plans;
+  const int rc = plan_batch(batch, p, &plans);
+  if (rc != VC_OK) return rc;
+  if (!Qw || !K || !V || !K_out || !V_out || !idx_out) return VC_ERR_INVALID_ARG;
+  if (!aligned16(Qw) || !aligned16(K) || !aligned16(V) || !aligned16(K_out) || !aligned16(V_out))
+    return VC_ERR_INVALID_ARG;
+  Layout lay = compress_layout(p, plans);
+  const int wc = check_ws(ws, ws_bytes, lay.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = lay.upload(w, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  const float scale = p->scale == 0.f ? 1.0f / sqrtf((float)p->d) : p->scale;
+  const Shape sh = lay.shape(scale);
+  const Tables tb = lay.tables(w);
+  float* scores = reinterpret_cast<float*>(w + lay.o_scores);
+  int32_t* rank = reinterpret_cast<int32_t*>(w + lay.o_rank);
+  int32_t* drop = reinterpret_cast<int32_t*>(w + lay.o_drop);
+  e = launch_score_simt(p->dtype, Qw, K, sh, tb, lay.units_lse, lay.units_col,
+                        reinterpret_cast<float*>(w + lay.o_lse), nullptr, scores, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  const int problems = lay.n_req * (p->rank_mode == VC_RANK_PER_LAYER ? p->L * p->Hkv : p->Hkv);
+  e = launch_select(sh, tb, problems, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
+                    reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  e = launch_gather_k(p->dtype, K, sh, tb, idx_out, K_out, lay.out_rows, st);
+  if (e != cudaSuccess) return VC_ERR_CUDA;
+  e = launch_fuse_simt(p->dtype, V, sh, tb, idx_out, drop, p->mu, p->tau, V_out, lay.units_fuse, st);
+  return cuda_status(e);
+}
+
+int prunekv_get_status(const void* ws, void* stream) {
+  if (!ws) return VC_ERR_WORKSPACE;
+  int32_t s = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&s, ws, sizeof(s), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return VC_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return VC_ERR_CUDA;
+  return s;
+}
+
+}  // extern "C"

@@ -1,0 +1,41 @@
+// Launchers of the libviscache kernels (internal; the C ABI is include/viscache.h).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "vc_common.cuh"
+
+namespace vc {
+
+// Plan-table image passed by value (kernel parameters may hold up to 32 KB).
+struct TableImage {
+  alignas(16) uint8_t bytes[24 * 1024];
+};
+cudaError_t launch_upload(const TableImage& im, uint32_t bytes, uint8_t* dst, int32_t* status,
+                          cudaStream_t st);
+
+int score_rows_per_tile_simt();
+int score_keys_per_tile_simt();
+int fuse_rows_per_tile_simt();
+
+// Eq. (token_score) on CUDA cores: lse pass (skipped when lse_nat != nullptr) + column sums.
+cudaError_t launch_score_simt(int dtype, const void* Qw, const void* K, const Shape& sh,
+                              const Tables& tb, int units_lse, int units_col, float* lse,
+                              const float* lse_nat, float* scores, cudaStream_t st);
+
+// Ranking (radix sort per problem) and ascending keep/drop compaction.
+cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, const float* scores,
+                          int32_t* rank, uint32_t* keys, int32_t* vals, int64_t sort_stride,
+                          int32_t* keep_idx, int32_t* drop_idx, cudaStream_t st);
+
+// K_out = K[keep] (bit-exact), total_rows = Hkv * sum over requests and layers of B_l.
+cudaError_t launch_gather_k(int dtype, const void* K, const Shape& sh, const Tables& tb,
+                            const int32_t* keep_idx, void* K_out, int64_t total_rows,
+                            cudaStream_t st);
+
+// V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on CUDA cores.
+cudaError_t launch_fuse_simt(int dtype, const void* V, const Shape& sh, const Tables& tb,
+                             const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
+                             void* V_out, int units, cudaStream_t st);
+
+}  // namespace vc

@@ -1,0 +1,287 @@
+"""Python binding of libviscache (include/viscache.h): argument marshalling only.
+
+Every function here has the name of the C entry point it calls.  torch is used
+for device memory (outputs and workspaces) and for the current CUDA stream;
+every step of the compression pass runs in the library's kernels.  There is no
+fallback: if ``_lib/libviscache.so`` is missing or fails to load, importing
+the functions raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence, Tuple
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libviscache.so")
+
+VC_OK = 0
+VC_ERR_INVALID_ARG = 1
+VC_ERR_INFEASIBLE = 2
+VC_ERR_WORKSPACE = 3
+VC_ERR_CUDA = 4
+VC_ERR_DEVICE_TIMEOUT = 5
+VC_ERR_UNSUPPORTED = 6
+VC_ERR_DEVICE_INDEX = 7
+VC_BF16, VC_F32 = 0, 1
+VC_RANK_SHARED, VC_RANK_PER_LAYER = 0, 1
+
+_ERR_NAMES = {1: "VC_ERR_INVALID_ARG", 2: "VC_ERR_INFEASIBLE", 3: "VC_ERR_WORKSPACE",
+              4: "VC_ERR_CUDA", 5: "VC_ERR_DEVICE_TIMEOUT", 6: "VC_ERR_UNSUPPORTED",
+              7: "VC_ERR_DEVICE_INDEX"}
+
+EXPORTED = ("viscache_plan_budgets", "prunekv_score_workspace_size", "prunekv_score",
+            "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
+            "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
+            "prunekv_get_status", "viscache_version", "viscache_profile_enable",
+            "viscache_profile_read")
+
+
+class VisCacheError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__("%s failed: %s (%d)" % (fn, _ERR_NAMES.get(code, "unknown"), code))
+        self.code = code
+
+
+class vc_batch(ctypes.Structure):
+    _fields_ = [("n_req", ctypes.c_int32), ("n_vis", ctypes.POINTER(ctypes.c_int32)),
+                ("W", ctypes.POINTER(ctypes.c_int32)), ("rr_num", ctypes.POINTER(ctypes.c_uint32)),
+                ("rr_den", ctypes.POINTER(ctypes.c_uint32))]
+
+
+class vc_params(ctypes.Structure):
+    _fields_ = [("L", ctypes.c_int32), ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32),
+                ("d", ctypes.c_int32), ("dtype", ctypes.c_int32), ("h", ctypes.c_int32),
+                ("m_num", ctypes.c_uint32), ("m_den", ctypes.c_uint32), ("mu", ctypes.c_float),
+                ("tau", ctypes.c_float), ("scale", ctypes.c_float), ("rank_mode", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library (loads on first use; raises if it was never built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError("libviscache.so is not built (%s); run __graft_entry__.build()" % _LIB_PATH)
+        L = ctypes.CDLL(_LIB_PATH)
+        vp, i32, u32, f32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint32, ctypes.c_float, ctypes.c_size_t
+        pi32 = ctypes.POINTER(ctypes.c_int32)
+        L.viscache_plan_budgets.argtypes = [i32, i32, u32, u32, i32, u32, u32, pi32, pi32, pi32]
+        L.prunekv_score_workspace_size.argtypes = [i32, i32, i32]
+        L.prunekv_score_workspace_size.restype = sz
+        L.prunekv_score.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp, vp,
+                                    vp, sz, vp]
+        L.prunekv_select_workspace_size.argtypes = [i32, i32, i32, i32]
+        L.prunekv_select_workspace_size.restype = sz
+        L.prunekv_select.argtypes = [vp, i32, i32, i32, pi32, i32, i32, vp, vp, vp, vp, sz, vp]
+        L.prunekv_fuse_workspace_size.argtypes = [i32]
+        L.prunekv_fuse_workspace_size.restype = sz
+        L.prunekv_fuse_compact.argtypes = [vp, vp, i32, i32, i32, i32, i32, pi32, i32, vp, vp, f32,
+                                           f32, vp, vp, vp, sz, vp]
+        L.prunekv_workspace_size.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params)]
+        L.prunekv_workspace_size.restype = sz
+        L.prunekv_compress.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), vp, vp,
+                                       vp, vp, vp, vp, vp, sz, vp]
+        L.prunekv_get_status.argtypes = [vp, vp]
+        L.viscache_version.restype = ctypes.c_char_p
+        L.viscache_profile_enable.argtypes = [i32]
+        L.viscache_profile_read.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(ctypes.c_float),
+                                            pi32, i32]
+        _lib = L
+    return _lib
+
+
+def _check(fn: str, rc: int) -> None:
+    if rc != VC_OK:
+        raise VisCacheError(fn, rc)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return VC_BF16
+    if t.dtype == torch.float32:
+        return VC_F32
+    raise TypeError("unsupported dtype %s (bf16 or fp32)" % t.dtype)
+
+
+def _workspace(nbytes: int, device, ws: Optional[torch.Tensor]) -> torch.Tensor:
+    if ws is not None:
+        return ws
+    return torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+
+
+def _i32(seq):
+    arr = (ctypes.c_int32 * len(seq))(*[int(x) for x in seq])
+    return arr
+
+
+# ---------------------------------------------------------------------------
+
+def viscache_version() -> str:
+    return lib().viscache_version().decode()
+
+
+def viscache_plan_budgets(L: int, n_vis: int, rr_num: int, rr_den: int, h: int = 0,
+                          m_num: int = 3, m_den: int = 4) -> Tuple[List[int], int, int]:
+    """Host planner (Eq. parabolic): returns (B[L], Nq, h)."""
+    B = (ctypes.c_int32 * L)()
+    nq, hh = ctypes.c_int32(), ctypes.c_int32()
+    _check("viscache_plan_budgets",
+           lib().viscache_plan_budgets(L, n_vis, rr_num, rr_den, h, m_num, m_den, B,
+                                       ctypes.byref(nq), ctypes.byref(hh)))
+    return list(B), nq.value, hh.value
+
+
+def prunekv_score_workspace_size(L: int, Hq: int, W: int) -> int:
+    return lib().prunekv_score_workspace_size(L, Hq, W)
+
+
+def prunekv_score(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,
+                  rank_mode: int = VC_RANK_SHARED, row_lse: Optional[torch.Tensor] = None,
+                  scores: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                  stream=None) -> torch.Tensor:
+    """Eq. (token_score): scores [Hkv][n] (shared) or [L][Hkv][n] (per layer), fp32."""
+    L, Hq, W, d = Qw.shape
+    _, Hkv, n, _ = K.shape
+    if scores is None:
+        shape = (Hkv, n) if rank_mode == VC_RANK_SHARED else (L, Hkv, n)
+        scores = torch.empty(shape, dtype=torch.float32, device=K.device)
+    ws = _workspace(prunekv_score_workspace_size(L, Hq, W), K.device, ws)
+    _check("prunekv_score", lib().prunekv_score(
+        _ptr(Qw), _ptr(K), _dtype_code(K), L, Hq, Hkv, d, n, W, float(scale), rank_mode,
+        _ptr(row_lse), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
+    return scores
+
+
+def prunekv_select_workspace_size(L: int, Hkv: int, n_vis: int, rank_mode: int = VC_RANK_SHARED) -> int:
+    return lib().prunekv_select_workspace_size(L, Hkv, n_vis, rank_mode)
+
+
+def drop_rows(B: Sequence[int], Nq: int, Hkv: int) -> int:
+    return Hkv * sum(Nq - b for b in B if b > 0)
+
+
+def prunekv_select(scores: torch.Tensor, B: Sequence[int], Nq: int, rank_mode: int = VC_RANK_SHARED,
+                   ws: Optional[torch.Tensor] = None, stream=None):
+    """Ranking and keep/drop lists: returns (rank, keep_idx, drop_idx), int32 device tensors."""
+    L = len(B)
+    Hkv, n = scores.shape[-2], scores.shape[-1]
+    dev = scores.device
+    rank = torch.empty(scores.shape, dtype=torch.int32, device=dev)
+    keep = torch.empty(max(1, Hkv * sum(B)), dtype=torch.int32, device=dev)
+    drop = torch.empty(max(1, drop_rows(B, Nq, Hkv)), dtype=torch.int32, device=dev)
+    ws = _workspace(prunekv_select_workspace_size(L, Hkv, n, rank_mode), dev, ws)
+    _check("prunekv_select", lib().prunekv_select(
+        _ptr(scores), L, Hkv, n, _i32(B), Nq, rank_mode, _ptr(rank), _ptr(keep), _ptr(drop),
+        _ptr(ws), ws.numel(), _stream(stream)))
+    return rank, keep[:Hkv * sum(B)], drop[:drop_rows(B, Nq, Hkv)]
+
+
+def prunekv_fuse_workspace_size(L: int) -> int:
+    return lib().prunekv_fuse_workspace_size(L)
+
+
+def prunekv_fuse_compact(K: torch.Tensor, V: torch.Tensor, B: Sequence[int], Nq: int,
+                         keep_idx: torch.Tensor, drop_idx: torch.Tensor, mu: float = 0.7,
+                         tau: float = 1.0, K_out: Optional[torch.Tensor] = None,
+                         V_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                         stream=None):
+    """Prune keys / fuse values (Eq. redistribution, Eq. weight_fusion): returns (K_out, V_out)."""
+    L, Hkv, n, d = K.shape
+    rows = Hkv * sum(B)
+    if K_out is None:
+        K_out = torch.empty((max(rows, 1), d), dtype=K.dtype, device=K.device)
+    if V_out is None:
+        V_out = torch.empty((max(rows, 1), d), dtype=V.dtype, device=V.device)
+    keep_idx = keep_idx if keep_idx.numel() else torch.zeros(1, dtype=torch.int32, device=K.device)
+    drop_idx = drop_idx if drop_idx.numel() else torch.zeros(1, dtype=torch.int32, device=K.device)
+    ws = _workspace(prunekv_fuse_workspace_size(L), K.device, ws)
+    _check("prunekv_fuse_compact", lib().prunekv_fuse_compact(
+        _ptr(K), _ptr(V), _dtype_code(K), L, Hkv, d, n, _i32(B), Nq, _ptr(keep_idx),
+        _ptr(drop_idx), float(mu), float(tau), _ptr(K_out), _ptr(V_out), _ptr(ws), ws.numel(),
+        _stream(stream)))
+    return K_out[:rows], V_out[:rows]
+
+
+class Batch:
+    """Host description of a batch (vc_batch) kept alive with its arrays."""
+
+    def __init__(self, n_vis: Sequence[int], W: Sequence[int], rr: Sequence[Tuple[int, int]]):
+        k = len(n_vis)
+        self._n = (ctypes.c_int32 * k)(*n_vis)
+        self._w = (ctypes.c_int32 * k)(*W)
+        self._a = (ctypes.c_uint32 * k)(*[a for a, _ in rr])
+        self._b = (ctypes.c_uint32 * k)(*[b for _, b in rr])
+        self.c = vc_batch(k, self._n, self._w, self._a, self._b)
+        self.n_vis, self.W, self.rr = list(n_vis), list(W), list(rr)
+
+
+def make_params(L: int, Hq: int, Hkv: int, d: int, dtype: int, h: int = 0, m=(3, 4),
+                mu: float = 0.7, tau: float = 1.0, scale: float = 0.0,
+                rank_mode: int = VC_RANK_SHARED) -> vc_params:
+    return vc_params(L, Hq, Hkv, d, dtype, h, m[0], m[1], mu, tau, scale, rank_mode)
+
+
+def prunekv_workspace_size(batch: Batch, params: vc_params) -> int:
+    return lib().prunekv_workspace_size(ctypes.byref(batch.c), ctypes.byref(params))
+
+
+def compressed_rows(batch: Batch, params: vc_params) -> int:
+    rows = 0
+    for n, (a, b) in zip(batch.n_vis, batch.rr):
+        B, _, _ = viscache_plan_budgets(params.L, n, a, b, params.h, params.m_num, params.m_den)
+        rows += params.Hkv * sum(B)
+    return rows
+
+
+def prunekv_compress(batch: Batch, params: vc_params, Qw: torch.Tensor, K: torch.Tensor,
+                     V: torch.Tensor, K_out: Optional[torch.Tensor] = None,
+                     V_out: Optional[torch.Tensor] = None, idx_out: Optional[torch.Tensor] = None,
+                     ws: Optional[torch.Tensor] = None, stream=None):
+    """The whole pass over a packed batch: returns (K_out, V_out, idx_out)."""
+    rows = compressed_rows(batch, params)
+    dev = K.device
+    if K_out is None:
+        K_out = torch.empty((max(rows, 1), params.d), dtype=K.dtype, device=dev)
+    if V_out is None:
+        V_out = torch.empty((max(rows, 1), params.d), dtype=V.dtype, device=dev)
+    if idx_out is None:
+        idx_out = torch.empty(max(rows, 1), dtype=torch.int32, device=dev)
+    ws = _workspace(prunekv_workspace_size(batch, params), dev, ws)
+    _check("prunekv_compress", lib().prunekv_compress(
+        ctypes.byref(batch.c), ctypes.byref(params), _ptr(Qw), _ptr(K), _ptr(V), _ptr(K_out),
+        _ptr(V_out), _ptr(idx_out), _ptr(ws), ws.numel(), _stream(stream)))
+    return K_out[:rows], V_out[:rows], idx_out[:rows]
+
+
+def viscache_profile_enable(on: bool) -> None:
+    _check("viscache_profile_enable", lib().viscache_profile_enable(1 if on else 0))
+
+
+def viscache_profile_read(max_kernels: int = 32):
+    """{kernel name: (total ms, launches)} recorded since profiling was enabled / last read."""
+    names = ctypes.create_string_buffer(4096)
+    ms = (ctypes.c_float * max_kernels)()
+    cnt = (ctypes.c_int32 * max_kernels)()
+    k = lib().viscache_profile_read(names, 4096, ms, cnt, max_kernels)
+    if k < 0:
+        raise VisCacheError("viscache_profile_read", -k)
+    keys = names.value.decode().split("\n")[:k]
+    return {keys[i]: (ms[i], cnt[i]) for i in range(k)}
+
+
+def prunekv_get_status(ws: torch.Tensor, stream=None) -> int:
+    return lib().prunekv_get_status(_ptr(ws), _stream(stream))

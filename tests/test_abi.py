@@ -1,0 +1,100 @@
+"""CPU checks of the C-ABI library: it loads, exports every declared symbol, the host
+planner matches the oracle planner bit-exactly, and argument errors come back as codes."""
+import ctypes
+import os
+import re
+from fractions import Fraction
+
+import pytest
+
+from oracle import plan
+from paper_2608_24063_gb300 import viscache as vc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "viscache.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:int|size_t|const char\*)\s+(\w+)\s*\(", src, flags=re.M)))
+
+
+def test_library_exports_every_declared_symbol():
+    names = _declared()
+    assert "prunekv_compress" in names and "viscache_plan_budgets" in names
+    lib = vc.lib()
+    for name in names:
+        assert hasattr(lib, name), name
+    assert set(vc.EXPORTED) == set(names)
+
+
+def test_version():
+    assert "sm_103a" in vc.viscache_version()
+
+
+@pytest.mark.parametrize("rr", [(19, 100), (22, 100), (23, 100), (28, 100), (1, 3), (56, 100)])
+def test_planner_matches_oracle_exhaustive_L(rr):
+    for L in range(1, 129):
+        for n in (1, 7, 1000, 3136, 12544, 32768):
+            try:
+                ref = plan.plan_budgets(L, n, Fraction(*rr))
+            except plan.Infeasible:
+                with pytest.raises(vc.VisCacheError) as ei:
+                    vc.viscache_plan_budgets(L, n, *rr)
+                assert ei.value.code == vc.VC_ERR_INFEASIBLE
+                continue
+            got = vc.viscache_plan_budgets(L, n, *rr)
+            assert got == (ref[0], ref[1], ref[2]), (L, n, rr)
+
+
+def test_planner_explicit_h_and_m():
+    for L, h, m in [(28, 14, (1, 2)), (80, 80, (1, 1)), (5, 1, (3, 4)), (64, 48, (3, 4))]:
+        ref = plan.plan_budgets(L, 5000, Fraction(1, 5), h=h, m=Fraction(*m))
+        assert vc.viscache_plan_budgets(L, 5000, 1, 5, h, *m) == ref
+
+
+def test_planner_argument_errors():
+    for args in [(0, 10, 1, 2), (3, 0, 1, 2), (3, 10, 0, 2), (3, 10, 3, 2), (3, 10, 1, 0)]:
+        with pytest.raises(vc.VisCacheError) as ei:
+            vc.viscache_plan_budgets(*args)
+        assert ei.value.code == vc.VC_ERR_INVALID_ARG
+    with pytest.raises(vc.VisCacheError):
+        vc.viscache_plan_budgets(4, 10, 1, 2, 5)          # h > L
+
+
+def test_entry_points_reject_bad_arguments_without_touching_the_device():
+    lib = vc.lib()
+    p = ctypes.c_void_p(256)
+    # d not in {64, 128}
+    assert lib.prunekv_score(p, p, 0, 1, 2, 1, 96, 10, 4, 0.0, 0, None, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    # Hq % Hkv != 0
+    assert lib.prunekv_score(p, p, 0, 1, 3, 2, 64, 10, 4, 0.0, 0, None, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    # misaligned pointer
+    q = ctypes.c_void_p(258)
+    assert lib.prunekv_score(q, p, 0, 1, 2, 1, 64, 10, 4, 0.0, 0, None, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    # workspace too small / misaligned
+    assert lib.prunekv_score(p, p, 0, 1, 2, 1, 64, 10, 4, 0.0, 0, None, p, p, 16, None) == vc.VC_ERR_WORKSPACE
+    assert lib.prunekv_score(p, p, 0, 1, 2, 1, 64, 10, 4, 0.0, 0, None, p, ctypes.c_void_p(272), 1 << 20, None) == vc.VC_ERR_WORKSPACE
+    # B_l > Nq, Nq > n
+    B = (ctypes.c_int32 * 2)(5, 3)
+    assert lib.prunekv_select(p, 2, 1, 10, B, 4, 0, p, p, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    assert lib.prunekv_select(p, 2, 1, 10, B, 11, 0, p, p, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    # mu out of range, tau <= 0
+    B2 = (ctypes.c_int32 * 1)(2)
+    assert lib.prunekv_fuse_compact(p, p, 0, 1, 1, 64, 10, B2, 4, p, p, 1.5, 1.0, p, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    assert lib.prunekv_fuse_compact(p, p, 0, 1, 1, 64, 10, B2, 4, p, p, 0.5, 0.0, p, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
+    # batch: infeasible retention surfaces as VC_ERR_INFEASIBLE
+    b = vc.Batch([10], [4], [(1, 1)])
+    prm = vc.make_params(4, 2, 1, 64, vc.VC_BF16, h=2, m=(1, 2))
+    assert lib.prunekv_compress(ctypes.byref(b.c), ctypes.byref(prm), p, p, p, p, p, p, p, 1 << 30, None) == vc.VC_ERR_INFEASIBLE
+
+
+def test_workspace_sizes_are_positive_and_aligned():
+    assert vc.prunekv_score_workspace_size(28, 28, 64) % 256 == 0
+    assert vc.prunekv_score_workspace_size(28, 28, 64) >= 28 * 28 * 64 * 4
+    assert vc.prunekv_select_workspace_size(28, 4, 12544) >= 2 * 8 * 4 * 12544
+    assert vc.prunekv_fuse_workspace_size(28) > 0
+    b = vc.Batch([12544], [64], [(19, 100)])
+    prm = vc.make_params(28, 28, 4, 128, vc.VC_BF16)
+    assert vc.prunekv_workspace_size(b, prm) > vc.prunekv_score_workspace_size(28, 28, 64)
+    assert vc.compressed_rows(b, prm) == 4 * 66734

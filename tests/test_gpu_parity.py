@@ -1,0 +1,185 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on the same seeded inputs."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import plan as oplan
+from oracle import prunekv as ok
+from paper_2608_24063_gb300 import synth
+from paper_2608_24063_gb300 import viscache as vc
+from tests.parity import check_request, np64
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+def _rand(shape, key, dtype):
+    x = synth.normal(key, 0, int(np.prod(shape)), "cpu").view(*shape)
+    return synth._round(x, dtype)
+
+
+def run_steps(Q, K, V, B, Nq, mu=0.7, tau=1.0, rank_mode=vc.VC_RANK_SHARED, row_lse=None):
+    s = vc.prunekv_score(Q, K, rank_mode=rank_mode, row_lse=row_lse)
+    rank, keep, drop = vc.prunekv_select(s, B, Nq, rank_mode)
+    Ko, Vo = vc.prunekv_fuse_compact(K, V, B, Nq, keep, drop, mu, tau)
+    torch.cuda.synchronize()
+    return dict(scores=s, rank=rank, keep=keep, drop=drop, K_out=Ko, V_out=Vo)
+
+
+SMALL = [
+    # L, Hq, Hkv, d, n, W, dtype, rr
+    (1, 2, 1, 64, 1, 1, torch.float32, (1, 1)),
+    (2, 4, 2, 64, 63, 3, torch.bfloat16, (1, 2)),
+    (3, 7, 1, 128, 129, 5, torch.bfloat16, (1, 4)),
+    (4, 8, 1, 128, 1000, 64, torch.bfloat16, (19, 100)),
+    (2, 8, 4, 64, 257, 32, torch.float32, (25, 100)),
+    (1, 1, 1, 128, 64, 1, torch.bfloat16, (1, 1)),
+    (5, 6, 2, 128, 700, 17, torch.float32, (28, 100)),
+]
+
+
+@pytest.mark.parametrize("case", SMALL)
+def test_small_shapes_step_api(case):
+    L, Hq, Hkv, d, n, W, dt, rr = case
+    key = hash(case[:6]) & 0xFFFFFFFF
+    Q = _rand((L, Hq, W, d), key + 1, dt)
+    K = _rand((L, Hkv, n, d), key + 2, dt)
+    V = _rand((L, Hkv, n, d), key + 3, dt)
+    B, Nq, h = vc.viscache_plan_budgets(L, n, *rr)
+    from fractions import Fraction
+    assert (B, Nq, h) == oplan.plan_budgets(L, n, Fraction(*rr))
+    out = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq)
+    log = check_request(Q, K, V, B, Nq, out, 0.7, 1.0)
+    assert len(log) <= 2, log
+
+
+@pytest.mark.parametrize("case", SMALL[1:5])
+def test_compress_equals_step_api(case):
+    L, Hq, Hkv, d, n, W, dt, rr = case
+    key = hash(case[:6]) & 0xFFFFFFFF
+    Q, K, V = (_rand(s, key + i, dt).to(DEV) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)], 1))
+    B, Nq, h = vc.viscache_plan_budgets(L, n, *rr)
+    ref = run_steps(Q, K, V, B, Nq)
+    batch = vc.Batch([n], [W], [rr])
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_F32 if dt == torch.float32 else vc.VC_BF16)
+    Ko, Vo, idx = vc.prunekv_compress(batch, prm, Q, K, V)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, ref["keep"]) and torch.equal(Ko, ref["K_out"]) and torch.equal(Vo, ref["V_out"])
+
+
+def test_mu_one_is_plain_pruning_bit_exact():
+    L, Hq, Hkv, d, n, W = 3, 4, 2, 128, 300, 8
+    Q, K, V = (_rand(s, 700 + i, torch.bfloat16).to(DEV) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 1, 4)
+    out = run_steps(Q, K, V, B, Nq, mu=1.0)
+    keep = out["keep"].long().cpu()
+    P = 0
+    for l in range(L):
+        for g in range(Hkv):
+            r0 = Hkv * P + g * B[l]
+            rows = V[l, g].cpu()[keep[r0:r0 + B[l]]]
+            assert torch.equal(out["V_out"][r0:r0 + B[l]].cpu(), rows)
+        P += B[l]
+
+
+def test_empty_drop_set_keeps_values():
+    # L = 1, m = 1: Nq = B_1, nothing to fuse.
+    L, Hq, Hkv, d, n, W = 1, 2, 1, 64, 200, 4
+    Q, K, V = (_rand(s, 800 + i, torch.float32).to(DEV) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 1, 4, 0, 1, 1)
+    assert Nq == B[0]
+    out = run_steps(Q, K, V, B, Nq)
+    assert out["drop"].numel() == 0
+    assert torch.equal(out["V_out"].cpu(), V[0, 0].cpu()[out["keep"].long().cpu()])
+
+
+def test_zero_queries_keep_first_positions():
+    L, Hq, Hkv, d, n, W = 2, 4, 2, 128, 500, 16
+    Q = torch.zeros((L, Hq, W, d), dtype=torch.bfloat16, device=DEV)
+    K, V = (_rand((L, Hkv, n, d), 900 + i, torch.bfloat16).to(DEV) for i in range(2))
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 1, 4)
+    out = run_steps(Q, K, V, B, Nq)
+    keep = out["keep"].cpu()
+    for g in range(Hkv):
+        assert keep[g * B[0]:(g + 1) * B[0]].tolist() == list(range(B[0]))
+    assert torch.allclose(out["scores"].cpu(), torch.full((Hkv, n), 2.0 * W / n), rtol=1e-6)
+
+
+def test_per_layer_ranking():
+    L, Hq, Hkv, d, n, W = 3, 6, 2, 128, 333, 9
+    Q, K, V = (_rand(s, 1000 + i, torch.bfloat16) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 3, 10)
+    out = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq, rank_mode=vc.VC_RANK_PER_LAYER)
+    assert out["scores"].shape == (L, Hkv, n)
+    check_request(Q, K, V, B, Nq, out, 0.7, 1.0, rank_mode="per_layer")
+
+
+def test_row_lse_input():
+    L, Hq, Hkv, d, n, W = 2, 4, 2, 64, 190, 6
+    Q, K, V = (_rand(s, 1100 + i, torch.float32) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
+    Qn, Kn = np64(Q), np64(K)
+    lse = np.empty((L, Hq, W))
+    for l in range(L):
+        for j in range(Hq):
+            x = (Qn[l, j] @ Kn[l, j // 2].T) / np.sqrt(d)
+            lse[l, j] = np.log(np.exp(x).sum(axis=1)) + 0.25    # a wider softmax domain
+    lse32 = torch.from_numpy(lse).float()
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 1, 4)
+    out = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq, row_lse=lse32.to(DEV))
+    check_request(Q, K, V, B, Nq, out, 0.7, 1.0, row_lse=lse32.double().numpy())
+
+
+def test_bad_index_sets_device_status():
+    # A keep list with an out-of-range position: the kernels skip it and record
+    # VC_ERR_DEVICE_INDEX; the context stays usable.
+    L, Hkv, d, n = 1, 1, 64, 50
+    K, V = (_rand((L, Hkv, n, d), 1200 + i, torch.float32).to(DEV) for i in range(2))
+    B, Nq = [4], 6
+    keep = torch.tensor([1, 2, 3, 999], dtype=torch.int32, device=DEV)
+    drop = torch.tensor([5, 6], dtype=torch.int32, device=DEV)
+    ws = torch.empty(vc.prunekv_fuse_workspace_size(L), dtype=torch.uint8, device=DEV)
+    vc.prunekv_fuse_compact(K, V, B, Nq, keep, drop, ws=ws)
+    assert vc.prunekv_get_status(ws) == vc.VC_ERR_DEVICE_INDEX
+    keep[3] = 4
+    vc.prunekv_fuse_compact(K, V, B, Nq, keep, drop, ws=ws)
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+
+
+# ---------------------------------------------------------------------------
+# The workloads at full size.
+
+def _workload_inputs(wid, device="cpu"):
+    wl = synth.WORKLOADS[wid]
+    qs, ks, vs = synth.generate(wl, device)
+    return wl, qs[0], ks[0], vs[0]
+
+
+@pytest.mark.parametrize("wid", [1, 2, 3])
+def test_workload_full_parity(wid):
+    wl, Q, K, V = _workload_inputs(wid)
+    req = wl.requests[0]
+    B, Nq, h = vc.viscache_plan_budgets(wl.L, req.n, req.rr_num, req.rr_den)
+    out = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq)
+    log = check_request(Q, K, V, B, Nq, out, 0.7, 1.0)
+    print("workload %d near-tie swaps: %s" % (wid, log))
+    # the fused entry point gives the same bits
+    batch = vc.Batch([req.n], [req.W], [(req.rr_num, req.rr_den)])
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_F32 if wl.dtype == "f32" else vc.VC_BF16)
+    Ko, Vo, idx = vc.prunekv_compress(batch, prm, Q.to(DEV), K.to(DEV), V.to(DEV))
+    torch.cuda.synchronize()
+    assert torch.equal(idx, out["keep"]) and torch.equal(Ko, out["K_out"]) and torch.equal(Vo, out["V_out"])
+
+
+def test_generator_same_bits_on_device():
+    wl = synth.scaled(synth.WORKLOADS[3], "slice", L=2)
+    q_cpu = synth.make_q(wl, 0, "cpu")
+    q_dev = synth.make_q(wl, 0, DEV)
+    assert torch.equal(q_cpu, q_dev.cpu())
+    k_cpu, v_cpu = synth.make_kv(wl, 0, q_cpu, "cpu", layers=[1])
+    k_dev, v_dev = synth.make_kv(wl, 0, q_cpu, DEV, layers=[1])
+    assert torch.equal(k_cpu[1], k_dev[1].cpu()) and torch.equal(v_cpu[1], v_dev[1].cpu())

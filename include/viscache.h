@@ -114,6 +114,34 @@ int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t H
                   void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * prunekv_score_static -- prunekv_score for callers that cannot allocate
+ * device memory (code running inside an allocator or memory-pool hook, a
+ * runtime that replays frozen CUDA graphs and hands out no workspace, an
+ * embedding host without a device allocator).  The paper has no counterpart:
+ * this is a deployment convenience, not a step of the method.
+ *
+ * Same arguments, arithmetic and result as prunekv_score, minus the
+ * workspace: the scratch (status word, plan tables, per-row log-sum-exp) is a
+ * fixed device array of VC_STATIC_SCRATCH_BYTES inside the library, which
+ * every GPU that loads the library holds until the process exits.
+ *   - Problems needing more scratch than that (prunekv_score_workspace_size
+ *     (L, Hq, W) > VC_STATIC_SCRATCH_BYTES, i.e. roughly L*Hq*W > 1,000,000
+ *     window rows) are rejected with VC_ERR_WORKSPACE before any device work.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current and caches it; make
+ *     that first call before capturing a stream.  Nothing is allocated.
+ *   - All calls on a device share the array and it keeps the last call's
+ *     contents; each call rewrites everything it reads.  Calls whose kernels
+ *     overlap on the GPU race on the array: serialise them.
+ *   - Device-side status is kept in the shared array and is not reported;
+ *     the return value covers arguments and launches.
+ */
+#define VC_STATIC_SCRATCH_BYTES (4u << 20)
+int prunekv_score_static(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq,
+                         int32_t Hkv, int32_t d, int32_t n_vis, int32_t W, float scale,
+                         int rank_mode, const float* row_lse, float* scores, void* stream);
+
+/*
  * prunekv_select -- rank, keep and drop sets, Algorithm 1 steps 1 and 3.
  *
  * Per KV head (per (layer, KV head) in VC_RANK_PER_LAYER) tokens are ordered

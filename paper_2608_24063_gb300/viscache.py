@@ -35,7 +35,7 @@ EXPORTED = ("viscache_plan_budgets", "prunekv_score_workspace_size", "prunekv_sc
             "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
-            "viscache_profile_read")
+            "viscache_profile_read", "prunekv_score_static")
 
 
 class VisCacheError(RuntimeError):
@@ -74,6 +74,8 @@ def lib() -> ctypes.CDLL:
         L.prunekv_score_workspace_size.restype = sz
         L.prunekv_score.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp, vp,
                                     vp, sz, vp]
+        L.prunekv_score_static.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp,
+                                           vp, vp]
         L.prunekv_select_workspace_size.argtypes = [i32, i32, i32, i32]
         L.prunekv_select_workspace_size.restype = sz
         L.prunekv_select.argtypes = [vp, i32, i32, i32, pi32, i32, i32, vp, vp, vp, vp, sz, vp]
@@ -163,6 +165,29 @@ def prunekv_score(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,
     _check("prunekv_score", lib().prunekv_score(
         _ptr(Qw), _ptr(K), _dtype_code(K), L, Hq, Hkv, d, n, W, float(scale), rank_mode,
         _ptr(row_lse), _ptr(scores), _ptr(ws), ws.numel(), _stream(stream)))
+    return scores
+
+
+STATIC_SCRATCH_BYTES = 4 << 20
+
+
+def prunekv_score_static(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,
+                         rank_mode: int = VC_RANK_SHARED, row_lse: Optional[torch.Tensor] = None,
+                         scores: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """prunekv_score with the library's fixed scratch array instead of a workspace.
+
+    For callers that cannot allocate device memory: the C entry point
+    allocates nothing (pass ``scores`` to keep this wrapper allocation-free
+    too).  Calls overlapping on the GPU race on the shared scratch.
+    """
+    L, Hq, W, d = Qw.shape
+    _, Hkv, n, _ = K.shape
+    if scores is None:
+        shape = (Hkv, n) if rank_mode == VC_RANK_SHARED else (L, Hkv, n)
+        scores = torch.empty(shape, dtype=torch.float32, device=K.device)
+    _check("prunekv_score_static", lib().prunekv_score_static(
+        _ptr(Qw), _ptr(K), _dtype_code(K), L, Hq, Hkv, d, n, W, float(scale), rank_mode,
+        _ptr(row_lse), _ptr(scores), _stream(stream)))
     return scores
 
 

@@ -238,6 +238,16 @@ int viscache_profile_enable(int on);
 int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* launches,
                           int max_kernels);
 
+/*
+ * Kernel path selection (process-wide, default VC_PATH_AUTO): AUTO scores
+ * bf16, d = 128 problems on the tcgen05 tensor cores and everything else on
+ * CUDA cores; VC_PATH_SIMT forces the CUDA-core kernels (fp32 FFMA) for every
+ * problem.  Both compute the same quantities; used to cross-check the paths.
+ */
+#define VC_PATH_AUTO 0
+#define VC_PATH_SIMT 1
+int viscache_set_kernel_path(int path);
+
 /* Version string of the library build. */
 const char* viscache_version(void);
 

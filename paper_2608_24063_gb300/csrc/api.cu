@@ -6,6 +6,8 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <algorithm>
+#include <atomic>
 #include <vector>
 
 #include "kernels.h"
@@ -15,6 +17,17 @@ namespace vc {
 namespace {
 
 constexpr size_t kAlign = 256;
+
+// Kernel path: VC_PATH_AUTO uses the tcgen05 score kernels for bf16, d = 128.
+std::atomic<int> g_path{VC_PATH_AUTO};
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    return 148;
+  return n;
+}
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Sequential carving of the caller workspace into 256-byte aligned regions.
@@ -37,13 +50,17 @@ struct Layout {
   // inputs
   int n_req = 0, L = 0, Hq = 0, Hkv = 0, d = 0, rank_mode = VC_RANK_SHARED;
   bool need_lse = false, need_scores = false, need_sort = false, need_drop = false;
+  // tensor-core score plan
+  int S = 1;
+  int64_t q_rows = 0, k_rows = 0, max_rows = 0;
+  std::vector<int32_t> u_tc1, u_tc2, base_tc1;
   // derived sizes
   int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
   int units_lse = 0, units_col = 0, units_fuse = 0;
   // workspace offsets
   size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
-         o_row0 = 0, table_begin = 0, table_end = 0, o_lse = 0, o_scores = 0, o_keys = 0,
-         o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
+         o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, table_begin = 0, table_end = 0, o_lse = 0,
+         o_part = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
   // host images
   std::vector<Req> req;
   std::vector<Layer> layer;
@@ -59,6 +76,10 @@ struct Layout {
     u_col.assign(n_req + 1, 0);
     u_fuse.assign((size_t)n_req * L + 1, 0);
     row0.assign((size_t)n_req * L + 1, 0);
+    u_tc1.assign(n_req + 1, 0);
+    u_tc2.assign(n_req + 1, 0);
+    base_tc1.assign(n_req, 0);
+    q_rows = k_rows = max_rows = 0;
     int64_t cu_n = 0, cu_w = 0;
     const int per_req_problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
     const int rows_tile = score_rows_per_tile_simt(), keys_tile = score_keys_per_tile_simt();
@@ -73,6 +94,14 @@ struct Layout {
       q.out_row0 = out_rows;
       q.drop_row0 = drop_rows;
       q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
+      q.C = (G * p.W + 127) / 128;
+      q.nrb = (G * p.W + 255) / 256;
+      q.tiles = (p.n + 127) / 128;
+      base_tc1[r] = L * Hkv * q.nrb;
+      u_tc2[r + 1] = u_tc2[r] + Hkv * q.tiles;
+      q_rows += (int64_t)L * Hq * p.W;
+      k_rows += (int64_t)L * Hkv * p.n;
+      max_rows = std::max<int64_t>(max_rows, (int64_t)L * Hq * p.W);
       u_lse[r + 1] = u_lse[r] + (G * p.W + rows_tile - 1) / rows_tile;
       u_col[r + 1] = u_col[r] + (p.n + keys_tile - 1) / keys_tile;
       int32_t P = 0, Qd = 0;
@@ -97,6 +126,7 @@ struct Layout {
     units_lse = u_lse[n_req];
     units_col = u_col[n_req];
     units_fuse = u_fuse[(size_t)n_req * L];
+    set_splits(1);
 
     Arena a;
     o_status = a.take(kAlign);
@@ -107,8 +137,13 @@ struct Layout {
     o_u_col = a.take(sizeof(int32_t) * u_col.size());
     o_u_fuse = a.take(sizeof(int32_t) * u_fuse.size());
     o_row0 = a.take(sizeof(int64_t) * row0.size());
+    o_u_tc1 = a.take(sizeof(int32_t) * u_tc1.size());
+    o_u_tc2 = a.take(sizeof(int32_t) * u_tc2.size());
     table_end = a.off;
-    if (need_lse) o_lse = a.take(sizeof(float) * lse_elems);
+    if (need_lse) {
+      o_lse = a.take(sizeof(float) * lse_elems);
+      o_part = a.take(sizeof(float2) * lse_elems * score_tc_max_splits());
+    }
     if (need_scores) o_scores = a.take(sizeof(float) * score_elems);
     if (need_sort) {
       o_keys = a.take(sizeof(uint32_t) * 2 * score_elems);
@@ -117,6 +152,36 @@ struct Layout {
     }
     if (need_drop) o_drop = a.take(sizeof(int32_t) * drop_rows);
     total = a.off;
+  }
+
+  // Key splits of the tensor-core lse pass: pick S in [1, max] that fills the
+  // last wave of CTAs best (one CTA per SM); ties go to the smaller S.
+  void set_splits(int s) {
+    S = s;
+    for (int r = 0; r < n_req; ++r) u_tc1[r + 1] = u_tc1[r] + base_tc1[r] * S;
+  }
+  void choose_splits(int nsm) {
+    int best = 1;
+    double best_eff = -1.0;
+    for (int s = 1; s <= score_tc_max_splits(); ++s) {
+      int64_t units = 0;
+      for (int r = 0; r < n_req; ++r) units += (int64_t)base_tc1[r] * s;
+      const int64_t waves = (units + nsm - 1) / nsm;
+      const double eff = (double)units / (double)(waves * nsm);
+      if (eff > best_eff + 1e-9) { best_eff = eff; best = s; }
+    }
+    set_splits(best);
+  }
+
+  TcPlan tc_plan() const {
+    TcPlan t;
+    t.units1 = u_tc1[n_req];
+    t.units2 = u_tc2[n_req];
+    t.S = S;
+    t.q_rows = q_rows;
+    t.k_rows = k_rows;
+    t.max_rows = max_rows;
+    return t;
   }
 
   // Copy the table image into the workspace and clear the status word.  Small
@@ -149,6 +214,8 @@ struct Layout {
     put(o_u_col, u_col.data(), sizeof(int32_t) * u_col.size());
     put(o_u_fuse, u_fuse.data(), sizeof(int32_t) * u_fuse.size());
     put(o_row0, row0.data(), sizeof(int64_t) * row0.size());
+    put(o_u_tc1, u_tc1.data(), sizeof(int32_t) * u_tc1.size());
+    put(o_u_tc2, u_tc2.data(), sizeof(int32_t) * u_tc2.size());
   }
 
   Tables tables(uint8_t* ws) const {
@@ -159,6 +226,8 @@ struct Layout {
     t.unit0_col = reinterpret_cast<const int32_t*>(ws + o_u_col);
     t.unit0_fuse = reinterpret_cast<const int32_t*>(ws + o_u_fuse);
     t.row0_out = reinterpret_cast<const int64_t*>(ws + o_row0);
+    t.unit0_tc1 = reinterpret_cast<const int32_t*>(ws + o_u_tc1);
+    t.unit0_tc2 = reinterpret_cast<const int32_t*>(ws + o_u_tc2);
     t.status = reinterpret_cast<int32_t*>(ws + o_status);
     return t;
   }
@@ -172,6 +241,23 @@ struct Layout {
     return s;
   }
 };
+
+// Eq. (token_score) through the tensor-core kernels (bf16, d = 128) or the CUDA-core ones.
+cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, float scale,
+                         uint8_t* w, const float* row_lse, float* scores, cudaStream_t st) {
+  const bool tc = g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128;
+  if (tc) lay.choose_splits(sm_count());
+  cudaError_t e = lay.upload(w, st);
+  if (e != cudaSuccess) return e;
+  const Shape sh = lay.shape(scale);
+  const Tables tb = lay.tables(w);
+  float* lse = reinterpret_cast<float*>(w + lay.o_lse);
+  if (tc)
+    return launch_score_tc(Qw, K, sh, tb, lay.tc_plan(), reinterpret_cast<float2*>(w + lay.o_part),
+                           lse, row_lse, scores, st);
+  return launch_score_simt(dtype, Qw, K, sh, tb, lay.units_lse, lay.units_col, lse, row_lse,
+                           scores, st);
+}
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -263,7 +349,13 @@ using namespace vc;
 
 extern "C" {
 
-const char* viscache_version(void) { return "viscache-gb300 0.1 (sm_103a)"; }
+const char* viscache_version(void) { return "viscache-gb300 0.2 (sm_103a)"; }
+
+int viscache_set_kernel_path(int path) {
+  if (path != VC_PATH_AUTO && path != VC_PATH_SIMT) return VC_ERR_INVALID_ARG;
+  g_path.store(path);
+  return VC_OK;
+}
 
 size_t prunekv_score_workspace_size(int32_t L, int32_t Hq, int32_t W) {
   if (L < 1 || L > 256 || Hq < 1 || W < 1) return 0;
@@ -285,11 +377,7 @@ int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t H
   if (wc != VC_OK) return wc;
   uint8_t* w = static_cast<uint8_t*>(ws);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  cudaError_t e = lay.upload(w, st);
-  if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_score_simt(dtype, Qw, K, lay.shape(scale), lay.tables(w), lay.units_lse,
-                        lay.units_col, reinterpret_cast<float*>(w + lay.o_lse), row_lse, scores, st);
-  return cuda_status(e);
+  return cuda_status(launch_score(dtype, Qw, K, lay, scale, w, row_lse, scores, st));
 }
 
 size_t prunekv_select_workspace_size(int32_t L, int32_t Hkv, int32_t n_vis, int rank_mode) {
@@ -369,17 +457,14 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   if (wc != VC_OK) return wc;
   uint8_t* w = static_cast<uint8_t*>(ws);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  cudaError_t e = lay.upload(w, st);
-  if (e != cudaSuccess) return VC_ERR_CUDA;
   const float scale = p->scale == 0.f ? 1.0f / sqrtf((float)p->d) : p->scale;
-  const Shape sh = lay.shape(scale);
-  const Tables tb = lay.tables(w);
   float* scores = reinterpret_cast<float*>(w + lay.o_scores);
   int32_t* rank = reinterpret_cast<int32_t*>(w + lay.o_rank);
   int32_t* drop = reinterpret_cast<int32_t*>(w + lay.o_drop);
-  e = launch_score_simt(p->dtype, Qw, K, sh, tb, lay.units_lse, lay.units_col,
-                        reinterpret_cast<float*>(w + lay.o_lse), nullptr, scores, st);
+  cudaError_t e = launch_score(p->dtype, Qw, K, lay, scale, w, nullptr, scores, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
+  const Shape sh = lay.shape(scale);
+  const Tables tb = lay.tables(w);
   const int problems = lay.n_req * (p->rank_mode == VC_RANK_PER_LAYER ? p->L * p->Hkv : p->Hkv);
   e = launch_select(sh, tb, problems, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
                     reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);

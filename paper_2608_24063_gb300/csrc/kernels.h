@@ -23,6 +23,21 @@ cudaError_t launch_score_simt(int dtype, const void* Qw, const void* K, const Sh
                               const Tables& tb, int units_lse, int units_col, float* lse,
                               const float* lse_nat, float* scores, cudaStream_t st);
 
+// Eq. (token_score) on tcgen05 tensor cores (bf16, d = 128): lse pass (skipped when
+// lse_nat != nullptr), merge of key splits, column sums.
+struct TcPlan {
+  int units1;        // CTAs of the lse pass (sum over requests of L*Hkv*nrb*S)
+  int units2;        // CTAs of the column-sum pass (sum of Hkv*tiles)
+  int S;             // key splits of the lse pass
+  int64_t q_rows;    // rows of the packed Qw tensor
+  int64_t k_rows;    // rows of the packed K tensor
+  int64_t max_rows;  // max over requests of L*Hq*W
+};
+int score_tc_max_splits();
+cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
+                            const TcPlan& tp, float2* part, float* lse2, const float* lse_nat,
+                            float* scores, cudaStream_t st);
+
 // Ranking (radix sort per problem) and ascending keep/drop compaction.
 cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, const float* scores,
                           int32_t* rank, uint32_t* keys, int32_t* vals, int64_t sort_stride,

@@ -1,0 +1,537 @@
+// Token scoring on the tcgen05 tensor cores, Eq. (token_score); bf16 inputs, d = 128.
+//
+// Per (request, layer, KV head) the G*W window rows (contiguous in Qw) meet
+// the n visual keys (contiguous in K).  Logits come from tcgen05.mma (bf16 x
+// bf16 -> fp32 in tensor memory), operands staged by TMA with 128-byte
+// swizzling.  The exact softmax column sum needs every row's normaliser
+// first, so the score takes two passes over the logits:
+//
+//   pass 1 (score_lse_tc)    rows in TMEM lanes: per row, running max and
+//                            compensated sum of exp2 over a range of key
+//                            tiles -> partial (m, z) per key split;
+//   merge  (lse_merge)       lse2 = m + log2 z over the splits (or the
+//                            caller's natural-log normaliser * log2 e);
+//   pass 2 (score_colsum_tc) keys in TMEM lanes: each thread owns one key and
+//                            sums exp2(x*scale*log2e - lse2[row]) over all
+//                            rows of all layers (compensated), s = sum / L.
+//
+// Warp roles in both passes (384 threads, one CTA per SM): warp 0 issues TMA,
+// warp 1 issues MMAs (one thread), warp 2 owns the tensor-memory allocation,
+// warps 4-7 and 8-11 are two consumer warpgroups.  Every wait is bounded: on a
+// timeout the CTA stops issuing, waits for its own copies and MMAs, frees its
+// tensor memory and records VC_ERR_DEVICE_TIMEOUT.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "kernels.h"
+#include "profile.h"
+#include "tc_common.cuh"
+#include "vc_common.cuh"
+
+namespace vc {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 384;
+constexpr uint32_t kTile = 128;                 // keys per tile, rows per block / chunk
+constexpr uint32_t kKBlockBytes = kTile * 128;  // 128 rows x 64 bf16
+constexpr uint32_t kTileBytes = 2 * kKBlockBytes;
+constexpr int kStages1 = 3;                     // K ring of pass 1
+constexpr int kQStages = 4;                     // Q ring of pass 2
+constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  const uint32_t a = smem_u32(p);
+  return p + ((1024u - (a & 1023u)) & 1023u);
+}
+
+// Wait bounded by time only (used when draining after an abort).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  int dummy = 0;
+  mbar_wait(bar, parity, &dummy);
+}
+
+// mbarrier wait whose outcome is the same for all 32 lanes (tcgen05.ld is a
+// warp-wide instruction, so a warp must never split on a wait).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
+// 16 consecutive TMEM columns of this thread's lane, as floats.
+__device__ __forceinline__ void tmem_cols16(uint32_t taddr, float (&x)[16]) {
+  uint32_t r[16];
+  tmem_ld16(taddr, r);
+  tmem_wait(r);
+#pragma unroll
+  for (int j = 0; j < 16; ++j) x[j] = __uint_as_float(r[j]);
+}
+
+__device__ __forceinline__ float sum16(const float (&e)[16]) {
+  float a[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) a[j] = e[2 * j] + e[2 * j + 1];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) a[j] = a[2 * j] + a[2 * j + 1];
+  return (a[0] + a[1]) + (a[2] + a[3]);
+}
+
+// ---------------------------------------------------------------------------
+// pass 1
+
+struct P1Smem {
+  uint8_t q[2][2][kKBlockBytes];          // [row block][K-block]
+  uint8_t k[kStages1][2][kKBlockBytes];   // [stage][K-block]
+  uint64_t q_full;
+  uint64_t k_full[kStages1], k_empty[kStages1];
+  uint64_t tm_full[2][2], tm_empty[2][2]; // [row block][slot]
+  uint64_t mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    Shape sh, Tables tb, int S, float2* __restrict__ part) {
+  extern __shared__ uint8_t smem_raw[];
+  P1Smem& sm = *reinterpret_cast<P1Smem*>(align1024(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int r = upper_index(tb.unit0_tc1, sh.n_req, (int32_t)blockIdx.x);
+  const Req rq = tb.req[r];
+  int u = blockIdx.x - tb.unit0_tc1[r];
+  const int s = u % S;
+  u /= S;
+  const int rbp = u % rq.nrb;
+  u /= rq.nrb;
+  const int g = u % sh.Hkv, l = u / sh.Hkv;
+  const int rows = sh.G * rq.W;
+  const int nblk = (rows - rbp * 256) > (int)kTile ? 2 : 1;   // row blocks with valid rows
+  const int tps = (rq.tiles + S - 1) / S;
+  const int t_begin = s * tps;
+  const int ntiles = max(0, min(rq.tiles, t_begin + tps) - t_begin);
+  const int qrow0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + rbp * 256;
+  const int krow0 = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n);
+
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.q_full, 1);
+    for (int i = 0; i < kStages1; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
+    for (int b = 0; b < 2; ++b)
+      for (int i = 0; i < 2; ++i) { mbar_init(&sm.tm_full[b][i], 1); mbar_init(&sm.tm_empty[b][i], kTile); }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = sm.tmem_base;
+  volatile int* abort = &sm.abort;
+
+  if (warp == 0 && lane == 0) {
+    // ---- TMA producer
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
+    mbar_arrive_expect_tx(&sm.q_full, nblk * kTileBytes);
+    for (int b = 0; b < nblk; ++b)
+      for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.q[b][kb], &tmQ, kb * 64, qrow0 + b * (int)kTile, &sm.q_full);
+    int issued = 0;
+    for (int i = 0; i < ntiles; ++i) {
+      const int st = i % kStages1;
+      if (!mbar_wait(&sm.k_empty[st], ((i / kStages1) & 1) ^ 1, abort)) break;
+      mbar_arrive_expect_tx(&sm.k_full[st], kTileBytes);
+      const int y = krow0 + (t_begin + i) * (int)kTile;
+      tma_load_2d(sm.k[st][0], &tmK, 0, y, &sm.k_full[st]);
+      tma_load_2d(sm.k[st][1], &tmK, 64, y, &sm.k_full[st]);
+      ++issued;
+    }
+    // every copy this CTA started has landed before the CTA may exit
+    drain_wait(&sm.q_full, 0);
+    for (int i = max(0, issued - kStages1); i < issued; ++i)
+      drain_wait(&sm.k_full[i % kStages1], (i / kStages1) & 1);
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer
+    const uint32_t idesc = idesc_bf16_f32(kTile, kTile);
+    bool ok = mbar_wait(&sm.q_full, 0, abort);
+    for (int i = 0; ok && i < ntiles; ++i) {
+      const int st = i % kStages1;
+      if (!mbar_wait(&sm.k_full[st], (i / kStages1) & 1, abort)) break;
+      tc_fence_after();
+      const int slot = i & 1;
+      const uint32_t use = (uint32_t)i >> 1;
+      for (int b = 0; b < nblk && ok; ++b) {
+        if (!mbar_wait(&sm.tm_empty[b][slot], (use & 1) ^ 1, abort)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d = tbase + (uint32_t)(b * 2 + slot) * kTile;
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_bf16(d, desc_sw128(smem_u32(sm.q[b][kb]) + k * 32),
+                     desc_sw128(smem_u32(sm.k[st][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
+        mma_commit(&sm.tm_full[b][slot]);
+      }
+      if (ok) mma_commit(&sm.k_empty[st]);
+    }
+    mma_commit(&sm.mma_done);
+    drain_wait(&sm.mma_done, 0);
+  } else if (warp >= 4) {
+    // ---- row statistics: one thread per row (= TMEM lane)
+    const int b = (warp - 4) >> 2;
+    const int lrow = ((warp & 3) << 5) + lane;
+    const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    const float s2 = sh.scale_log2;
+    float m = -INFINITY;
+    Kahan z;
+    z.init();
+    for (int i = 0; b < nblk && i < ntiles; ++i) {
+      const int slot = i & 1;
+      const uint32_t use = (uint32_t)i >> 1;
+      if (!warp_wait(&sm.tm_full[b][slot], use & 1, abort)) break;
+      tc_fence_after();
+      const int valid = min((int)kTile, rq.n - (t_begin + i) * (int)kTile);
+      const uint32_t col0 = tbase + lane_off + (uint32_t)(b * 2 + slot) * kTile;
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {            // two halves of 64 columns
+        float x[4][16];
+#pragma unroll
+        for (int p = 0; p < 4; ++p) tmem_cols16(col0 + h * 64 + p * 16, x[p]);
+        if (h == 1) {
+          tc_fence_before();
+          mbar_arrive(&sm.tm_empty[b][slot]);   // columns copied out: the MMA may reuse them
+        }
+        float cm = -INFINITY;
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            if (h * 64 + p * 16 + j >= valid) x[p][j] = -INFINITY;
+            cm = fmaxf(cm, x[p][j]);
+          }
+        const float xm = cm * s2;
+        if (xm > m) {
+          const float c = exp2f(m - xm);
+          z.s *= c;
+          z.c *= c;
+          m = xm;
+        }
+        if (m != -INFINITY) {
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            float e[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) e[j] = exp2f(fmaf(x[p][j], s2, -m));
+            z.add(sum16(e));
+          }
+        }
+      }
+    }
+    const int rho = rbp * 256 + b * (int)kTile + lrow;
+    if (rho < rows)
+      part[(rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho) * S + s] = make_float2(m, z.s);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+  if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+}
+
+// ---------------------------------------------------------------------------
+// merge: lse2 per window row; grid (rows / 256, n_req)
+
+__global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __restrict__ part,
+                                 const float* __restrict__ lse_nat, float* __restrict__ lse2) {
+  const Req rq = tb.req[blockIdx.y];
+  const int64_t per = (int64_t)sh.L * sh.Hq * rq.W;
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= per) return;
+  const int64_t o = rq.lse_off + i;
+  if (lse_nat) {
+    lse2[o] = lse_nat[o] * kLog2e;
+    return;
+  }
+  float m = -INFINITY;
+  for (int s = 0; s < S; ++s) m = fmaxf(m, part[o * S + s].x);
+  float z = 0.f;
+  for (int s = 0; s < S; ++s) {
+    const float2 p = part[o * S + s];
+    if (p.x != -INFINITY) z += p.y * exp2f(p.x - m);
+  }
+  lse2[o] = m + log2f(z);
+}
+
+// ---------------------------------------------------------------------------
+// pass 2
+
+struct P2Smem {
+  uint8_t k[2][2][kKBlockBytes];          // [stage = layer & 1][K-block]
+  uint8_t q[kQStages][2][kKBlockBytes];   // [stage][K-block]
+  float lse[2][2][kTile];                 // [warpgroup][buffer][row]
+  float red[2][kTile];                    // [warpgroup][key]
+  uint64_t k_full[2], k_empty[2];
+  uint64_t q_full[kQStages], q_empty[kQStages];
+  uint64_t tm_full[kQStages], tm_empty[kQStages];
+  uint64_t mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+// MMA columns of chunk c: the remaining rows rounded up to a multiple of 16.
+__device__ __forceinline__ int chunk_cols(int rows, int c) {
+  const int left = min((int)kTile, rows - c * (int)kTile);
+  return (left + 15) & ~15;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                       Shape sh, Tables tb, const float* __restrict__ lse2, float* __restrict__ scores) {
+  extern __shared__ uint8_t smem_raw[];
+  P2Smem& sm = *reinterpret_cast<P2Smem*>(align1024(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int r = upper_index(tb.unit0_tc2, sh.n_req, (int32_t)blockIdx.x);
+  const Req rq = tb.req[r];
+  const int u = blockIdx.x - tb.unit0_tc2[r];
+  const int g = u / rq.tiles, kt = u % rq.tiles;
+  const int rows = sh.G * rq.W;
+  const int C = rq.C;
+  const int L = sh.L;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
+    for (int i = 0; i < kQStages; ++i) {
+      mbar_init(&sm.q_full[i], 1);
+      mbar_init(&sm.q_empty[i], 1);
+      mbar_init(&sm.tm_full[i], 1);
+      mbar_init(&sm.tm_empty[i], kTile);
+    }
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 2) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = sm.tmem_base;
+  volatile int* abort = &sm.abort;
+
+  if (warp == 0 && lane == 0) {
+    // ---- TMA producer: K tile of layer l, then the C row chunks of layer l
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
+    int k_issued = 0, q_issued = 0;
+    bool ok = true;
+    for (int l = 0; ok && l < L; ++l) {
+      const int ks = l & 1;
+      if (!mbar_wait(&sm.k_empty[ks], ((l >> 1) & 1) ^ 1, abort)) break;
+      mbar_arrive_expect_tx(&sm.k_full[ks], kTileBytes);
+      const int ky = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + kt * (int)kTile;
+      tma_load_2d(sm.k[ks][0], &tmK, 0, ky, &sm.k_full[ks]);
+      tma_load_2d(sm.k[ks][1], &tmK, 64, ky, &sm.k_full[ks]);
+      ++k_issued;
+      const int qy0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W);
+      for (int c = 0; c < C; ++c) {
+        const int q = l * C + c, qs = q % kQStages;
+        if (!mbar_wait(&sm.q_empty[qs], ((q / kQStages) & 1) ^ 1, abort)) { ok = false; break; }
+        mbar_arrive_expect_tx(&sm.q_full[qs], kTileBytes);
+        tma_load_2d(sm.q[qs][0], &tmQ, 0, qy0 + c * (int)kTile, &sm.q_full[qs]);
+        tma_load_2d(sm.q[qs][1], &tmQ, 64, qy0 + c * (int)kTile, &sm.q_full[qs]);
+        ++q_issued;
+      }
+    }
+    for (int i = max(0, k_issued - 2); i < k_issued; ++i) drain_wait(&sm.k_full[i & 1], (i >> 1) & 1);
+    for (int i = max(0, q_issued - kQStages); i < q_issued; ++i)
+      drain_wait(&sm.q_full[i % kQStages], (i / kQStages) & 1);
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer: D[key][row] = K_tile . Q_chunk^T
+    bool ok = true;
+    for (int l = 0; ok && l < L; ++l) {
+      const int ks = l & 1;
+      if (!mbar_wait(&sm.k_full[ks], (l >> 1) & 1, abort)) break;
+      for (int c = 0; c < C; ++c) {
+        const int q = l * C + c, qs = q % kQStages;
+        const uint32_t use = (uint32_t)(q / kQStages);
+        if (!mbar_wait(&sm.q_full[qs], use & 1, abort)) { ok = false; break; }
+        if (!mbar_wait(&sm.tm_empty[qs], (use & 1) ^ 1, abort)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t idesc = idesc_bf16_f32(kTile, (uint32_t)chunk_cols(rows, c));
+        const uint32_t d = tbase + (uint32_t)qs * kTile;
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_bf16(d, desc_sw128(smem_u32(sm.k[ks][kb]) + k * 32),
+                     desc_sw128(smem_u32(sm.q[qs][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
+        mma_commit(&sm.tm_full[qs]);
+        mma_commit(&sm.q_empty[qs]);
+      }
+      if (ok) mma_commit(&sm.k_empty[ks]);
+    }
+    mma_commit(&sm.mma_done);
+    drain_wait(&sm.mma_done, 0);
+  } else if (warp >= 4) {
+    // ---- column sums: one thread per key (= TMEM lane); warpgroup wg takes
+    // the chunks q = l*C + c with q % 2 == wg
+    const int wg = (warp - 4) >> 2;
+    const int key = ((warp & 3) << 5) + lane;
+    const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    const float s2 = sh.scale_log2;
+    const int v = kt * (int)kTile + key;
+    const bool per_layer = sh.rank_mode == VC_RANK_PER_LAYER;
+    const int nq = L * C;
+    auto lse_of = [&](int q) -> float {
+      const int l = q / C, c = q % C;
+      const int rho = c * (int)kTile + key;
+      return rho < rows ? lse2[rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho] : INFINITY;
+    };
+    float nxt = wg < nq ? lse_of(wg) : INFINITY;
+    Kahan tot, lay;
+    tot.init();
+    lay.init();
+    int n_mine = 0;
+    for (int q = 0; q < nq; ++q) {
+      const int l = q / C, c = q % C;
+      if ((q & 1) == wg) {
+        // stage this chunk's normalisers for the whole warpgroup
+        float* buf = sm.lse[wg][n_mine & 1];
+        buf[key] = nxt;
+        named_sync(2 + wg, kTile);
+        if (q + 2 < nq) nxt = lse_of(q + 2);
+        ++n_mine;
+        const int qs = q % kQStages;
+        const uint32_t use = (uint32_t)(q / kQStages);
+        const bool go = __all_sync(0xffffffffu, *abort == 0);
+        if (go && warp_wait(&sm.tm_full[qs], use & 1, abort)) {
+          tc_fence_after();
+          const int ncol = chunk_cols(rows, c);
+          const uint32_t col0 = tbase + lane_off + (uint32_t)qs * kTile;
+          for (int p0 = 0; p0 < ncol; p0 += 64) {
+            const int np = min(4, (ncol - p0) >> 4);
+            float x[4][16];
+#pragma unroll
+            for (int p = 0; p < 4; ++p)
+              if (p < np) tmem_cols16(col0 + p0 + p * 16, x[p]);
+            if (p0 + 64 >= ncol) {
+              tc_fence_before();
+              mbar_arrive(&sm.tm_empty[qs]);
+            }
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+              if (p < np) {
+                float e[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) e[j] = exp2f(fmaf(x[p][j], s2, -buf[p0 + p * 16 + j]));
+                lay.add(sum16(e));
+              }
+            }
+          }
+        }
+      }
+      if (c == C - 1) {
+        if (per_layer) {
+          sm.red[wg][key] = lay.s;
+          named_sync(1, 2 * kTile);
+          if (wg == 0 && v < rq.n)
+            scores[rq.s_off + ((int64_t)l * sh.Hkv + g) * rq.n + v] = sm.red[0][key] + sm.red[1][key];
+          named_sync(1, 2 * kTile);
+        } else {
+          tot.add(lay.s);
+        }
+        lay.init();
+      }
+    }
+    if (!per_layer) {
+      sm.red[wg][key] = tot.s;
+      named_sync(1, 2 * kTile);
+      if (wg == 0 && v < rq.n)
+        scores[rq.s_off + (int64_t)g * rq.n + v] = (sm.red[0][key] + sm.red[1][key]) / (float)L;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+  if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// [rows][128] bf16 tensor, boxes of 128 rows x 64 elements, 128-byte swizzle.
+bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc || rows == 0 || rows > 0x7fffffffull) return false;
+  cuuint64_t dims[2] = {128, rows};
+  cuuint64_t strides[1] = {256};
+  cuuint32_t box[2] = {64, kTile};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+int score_tc_max_splits() { return 2; }
+
+cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
+                            const TcPlan& tp, float2* part, float* lse2, const float* lse_nat,
+                            float* scores, cudaStream_t st) {
+  CUtensorMap mq, mk;
+  if (!make_rows_map(&mq, Qw, tp.q_rows) || !make_rows_map(&mk, K, tp.k_rows))
+    return cudaErrorInvalidValue;
+  cudaError_t e;
+  if (!lse_nat) {
+    const size_t smem1 = sizeof(P1Smem) + 1024;
+    e = cudaFuncSetAttribute(score_lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+    if (e != cudaSuccess) return e;
+    ProfileScope ps("score_lse_tc", st);
+    score_lse_tc_kernel<<<tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  {
+    ProfileScope ps("lse_merge", st);
+    lse_merge_kernel<<<dim3((unsigned)((tp.max_rows + 255) / 256), sh.n_req), 256, 0, st>>>(
+        sh, tb, tp.S, part, lse_nat, lse2);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  const size_t smem2 = sizeof(P2Smem) + 1024;
+  e = cudaFuncSetAttribute(score_colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+  if (e != cudaSuccess) return e;
+  ProfileScope ps("score_colsum_tc", st);
+  score_colsum_tc_kernel<<<tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, lse2, scores);
+  return cudaGetLastError();
+}
+
+}  // namespace vc

@@ -21,6 +21,10 @@ struct Req {                 // one request of a batch
   int64_t out_row0;          // first output row (K_out/V_out/idx_out)
   int64_t drop_row0;         // first drop-list row
   int32_t n, W, Nq, h;
+  int32_t C;                 // 128-row chunks of one (layer, KV head) row set, ceil(G*W/128)
+  int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
+  int32_t tiles;             // 128-key tiles, ceil(n/128)
+  int32_t pad_;
 };
 
 struct Layer {               // one (request, layer)
@@ -44,6 +48,8 @@ struct Tables {              // device pointers into the workspace
   const int32_t* unit0_col;  // [n_req + 1] key-tile units of the column-sum pass
   const int32_t* unit0_fuse; // [n_req * L + 1] kept-row-tile units x Hkv of the fusion
   const int64_t* row0_out;   // [n_req * L + 1] first output row of each (request, layer)
+  const int32_t* unit0_tc1;  // [n_req + 1] CTAs of the tensor-core lse pass
+  const int32_t* unit0_tc2;  // [n_req + 1] CTAs of the tensor-core column-sum pass
   int32_t* status;           // device status word
 };
 

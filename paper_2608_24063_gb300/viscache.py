@@ -26,6 +26,7 @@ VC_ERR_UNSUPPORTED = 6
 VC_ERR_DEVICE_INDEX = 7
 VC_BF16, VC_F32 = 0, 1
 VC_RANK_SHARED, VC_RANK_PER_LAYER = 0, 1
+VC_PATH_AUTO, VC_PATH_SIMT = 0, 1
 
 _ERR_NAMES = {1: "VC_ERR_INVALID_ARG", 2: "VC_ERR_INFEASIBLE", 3: "VC_ERR_WORKSPACE",
               4: "VC_ERR_CUDA", 5: "VC_ERR_DEVICE_TIMEOUT", 6: "VC_ERR_UNSUPPORTED",
@@ -35,7 +36,7 @@ EXPORTED = ("viscache_plan_budgets", "prunekv_score_workspace_size", "prunekv_sc
             "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
-            "viscache_profile_read", "prunekv_score_static")
+            "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path")
 
 
 class VisCacheError(RuntimeError):
@@ -90,6 +91,7 @@ def lib() -> ctypes.CDLL:
         L.prunekv_get_status.argtypes = [vp, vp]
         L.viscache_version.restype = ctypes.c_char_p
         L.viscache_profile_enable.argtypes = [i32]
+        L.viscache_set_kernel_path.argtypes = [i32]
         L.viscache_profile_read.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(ctypes.c_float),
                                             pi32, i32]
         _lib = L
@@ -290,6 +292,11 @@ def prunekv_compress(batch: Batch, params: vc_params, Qw: torch.Tensor, K: torch
         ctypes.byref(batch.c), ctypes.byref(params), _ptr(Qw), _ptr(K), _ptr(V), _ptr(K_out),
         _ptr(V_out), _ptr(idx_out), _ptr(ws), ws.numel(), _stream(stream)))
     return K_out[:rows], V_out[:rows], idx_out[:rows]
+
+
+def viscache_set_kernel_path(path: int) -> None:
+    """VC_PATH_AUTO (tensor cores for bf16, d=128) or VC_PATH_SIMT (CUDA cores everywhere)."""
+    _check("viscache_set_kernel_path", lib().viscache_set_kernel_path(path))
 
 
 def viscache_profile_enable(on: bool) -> None:

@@ -18,6 +18,13 @@ def _rand(shape, key, dtype):
     return synth._round(x, dtype)
 
 
+@pytest.fixture(params=[vc.VC_PATH_AUTO, vc.VC_PATH_SIMT], ids=["auto", "simt"])
+def kernel_path(request):
+    vc.viscache_set_kernel_path(request.param)
+    yield request.param
+    vc.viscache_set_kernel_path(vc.VC_PATH_AUTO)
+
+
 def run_steps(Q, K, V, B, Nq, mu=0.7, tau=1.0, rank_mode=vc.VC_RANK_SHARED, row_lse=None):
     s = vc.prunekv_score(Q, K, rank_mode=rank_mode, row_lse=row_lse)
     rank, keep, drop = vc.prunekv_select(s, B, Nq, rank_mode)
@@ -39,7 +46,7 @@ SMALL = [
 
 
 @pytest.mark.parametrize("case", SMALL)
-def test_small_shapes_step_api(case):
+def test_small_shapes_step_api(case, kernel_path):
     L, Hq, Hkv, d, n, W, dt, rr = case
     key = hash(case[:6]) & 0xFFFFFFFF
     Q = _rand((L, Hq, W, d), key + 1, dt)
@@ -96,7 +103,7 @@ def test_empty_drop_set_keeps_values():
     assert torch.equal(out["V_out"].cpu(), V[0, 0].cpu()[out["keep"].long().cpu()])
 
 
-def test_zero_queries_keep_first_positions():
+def test_zero_queries_keep_first_positions(kernel_path):
     L, Hq, Hkv, d, n, W = 2, 4, 2, 128, 500, 16
     Q = torch.zeros((L, Hq, W, d), dtype=torch.bfloat16, device=DEV)
     K, V = (_rand((L, Hkv, n, d), 900 + i, torch.bfloat16).to(DEV) for i in range(2))
@@ -108,7 +115,7 @@ def test_zero_queries_keep_first_positions():
     assert torch.allclose(out["scores"].cpu(), torch.full((Hkv, n), 2.0 * W / n), rtol=1e-6)
 
 
-def test_per_layer_ranking():
+def test_per_layer_ranking(kernel_path):
     L, Hq, Hkv, d, n, W = 3, 6, 2, 128, 333, 9
     Q, K, V = (_rand(s, 1000 + i, torch.bfloat16) for i, s in
                enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
@@ -118,7 +125,7 @@ def test_per_layer_ranking():
     check_request(Q, K, V, B, Nq, out, 0.7, 1.0, rank_mode="per_layer")
 
 
-def test_row_lse_input():
+def test_row_lse_input(kernel_path):
     L, Hq, Hkv, d, n, W = 2, 4, 2, 64, 190, 6
     Q, K, V = (_rand(s, 1100 + i, torch.float32) for i, s in
                enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)]))
@@ -150,6 +157,41 @@ def test_bad_index_sets_device_status():
     assert vc.prunekv_get_status(ws) == vc.VC_OK
 
 
+TC_SHAPES = [
+    # L, Hq, Hkv, n, W  (bf16, d = 128: the tensor-core score path)
+    (1, 1, 1, 1, 1),
+    (2, 7, 1, 127, 5),
+    (2, 8, 1, 129, 16),
+    (1, 2, 1, 128, 64),
+    (3, 14, 2, 1000, 19),     # 7*19 = 133 rows: two row blocks, ragged
+    (2, 28, 4, 300, 64),      # 448 rows per group
+    (1, 8, 1, 2049, 40),      # 320 rows: two 256-row blocks
+    (2, 4, 4, 513, 3),        # G = 1
+]
+
+
+@pytest.mark.parametrize("shape", TC_SHAPES)
+@pytest.mark.parametrize("mode", [vc.VC_RANK_SHARED, vc.VC_RANK_PER_LAYER], ids=["shared", "layer"])
+def test_tensor_core_scores_match_oracle_and_cuda_cores(shape, mode):
+    L, Hq, Hkv, n, W = shape
+    d = 128
+    key = 5000 + 13 * sum(shape)
+    Q = _rand((L, Hq, W, d), key, torch.bfloat16)
+    K = _rand((L, Hkv, n, d), key + 1, torch.bfloat16)
+    Qd, Kd = Q.to(DEV), K.to(DEV)
+    s_tc = vc.prunekv_score(Qd, Kd, rank_mode=mode)
+    vc.viscache_set_kernel_path(vc.VC_PATH_SIMT)
+    try:
+        s_simt = vc.prunekv_score(Qd, Kd, rank_mode=mode)
+    finally:
+        vc.viscache_set_kernel_path(vc.VC_PATH_AUTO)
+    torch.cuda.synchronize()
+    ref = ok.token_scores(np64(Q), np64(K), rank_mode="per_layer" if mode else "shared")
+    for got in (s_tc, s_simt):
+        err = np.abs(np64(got) - ref) / np.maximum(np.abs(ref), 1e-30)
+        assert float(err.max()) < 2e-5, float(err.max())
+
+
 # ---------------------------------------------------------------------------
 # The workloads at full size.
 
@@ -160,7 +202,9 @@ def _workload_inputs(wid, device="cpu"):
 
 
 @pytest.mark.parametrize("wid", [1, 2, 3])
-def test_workload_full_parity(wid):
+def test_workload_full_parity(wid, kernel_path):
+    if wid == 1 and kernel_path == vc.VC_PATH_SIMT:
+        pytest.skip("fp32 workload runs on CUDA cores under both settings")
     wl, Q, K, V = _workload_inputs(wid)
     req = wl.requests[0]
     B, Nq, h = vc.viscache_plan_budgets(wl.L, req.n, req.rr_num, req.rr_den)

@@ -239,10 +239,11 @@ int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* lau
                           int max_kernels);
 
 /*
- * Kernel path selection (process-wide, default VC_PATH_AUTO): AUTO scores
- * bf16, d = 128 problems on the tcgen05 tensor cores and everything else on
- * CUDA cores; VC_PATH_SIMT forces the CUDA-core kernels (fp32 FFMA) for every
- * problem.  Both compute the same quantities; used to cross-check the paths.
+ * Kernel path selection (process-wide, default VC_PATH_AUTO): AUTO runs the
+ * score (Eq. token_score) and the fusion (Eq. redistribution, weight_fusion)
+ * of bf16, d = 128 problems on the tcgen05 tensor cores and everything else
+ * on CUDA cores; VC_PATH_SIMT forces the CUDA-core kernels (fp32 FFMA) for
+ * every problem.  Both compute the same quantities; used to cross-check.
  */
 #define VC_PATH_AUTO 0
 #define VC_PATH_SIMT 1

@@ -53,13 +53,14 @@ struct Layout {
   // tensor-core score plan
   int S = 1;
   int64_t q_rows = 0, k_rows = 0, max_rows = 0;
-  std::vector<int32_t> u_tc1, u_tc2, base_tc1;
+  std::vector<int32_t> u_tc1, u_tc2, base_tc1, u_fuse_tc;
+  int units_fuse_tc = 0;
   // derived sizes
   int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
   int units_lse = 0, units_col = 0, units_fuse = 0;
   // workspace offsets
   size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
-         o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, table_begin = 0, table_end = 0, o_lse = 0,
+         o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, o_u_fuse_tc = 0, table_begin = 0, table_end = 0, o_lse = 0,
          o_part = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
   // host images
   std::vector<Req> req;
@@ -77,6 +78,7 @@ struct Layout {
     u_fuse.assign((size_t)n_req * L + 1, 0);
     row0.assign((size_t)n_req * L + 1, 0);
     u_tc1.assign(n_req + 1, 0);
+    u_fuse_tc.assign((size_t)n_req * L + 1, 0);
     u_tc2.assign(n_req + 1, 0);
     base_tc1.assign(n_req, 0);
     q_rows = k_rows = max_rows = 0;
@@ -84,6 +86,7 @@ struct Layout {
     const int per_req_problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
     const int rows_tile = score_rows_per_tile_simt(), keys_tile = score_keys_per_tile_simt();
     const int fuse_tile = fuse_rows_per_tile_simt();
+    const int fuse_tile_tc = fuse_rows_per_tile_tc();
     for (int r = 0; r < n_req; ++r) {
       const RequestPlan& p = plans[r];
       Req& q = req[r];
@@ -112,6 +115,7 @@ struct Layout {
         ly.B = b; ly.P = P; ly.D = b > 0 ? p.Nq - b : 0; ly.Qd = Qd;
         row0[rl] = out_rows + (int64_t)Hkv * P;
         u_fuse[rl + 1] = u_fuse[rl] + Hkv * ((b + fuse_tile - 1) / fuse_tile);
+        u_fuse_tc[rl + 1] = u_fuse_tc[rl] + Hkv * ((b + fuse_tile_tc - 1) / fuse_tile_tc);
         P += b;
         Qd += ly.D;
       }
@@ -126,6 +130,7 @@ struct Layout {
     units_lse = u_lse[n_req];
     units_col = u_col[n_req];
     units_fuse = u_fuse[(size_t)n_req * L];
+    units_fuse_tc = u_fuse_tc[(size_t)n_req * L];
     set_splits(1);
 
     Arena a;
@@ -139,6 +144,7 @@ struct Layout {
     o_row0 = a.take(sizeof(int64_t) * row0.size());
     o_u_tc1 = a.take(sizeof(int32_t) * u_tc1.size());
     o_u_tc2 = a.take(sizeof(int32_t) * u_tc2.size());
+    o_u_fuse_tc = a.take(sizeof(int32_t) * u_fuse_tc.size());
     table_end = a.off;
     if (need_lse) {
       o_lse = a.take(sizeof(float) * lse_elems);
@@ -216,6 +222,7 @@ struct Layout {
     put(o_row0, row0.data(), sizeof(int64_t) * row0.size());
     put(o_u_tc1, u_tc1.data(), sizeof(int32_t) * u_tc1.size());
     put(o_u_tc2, u_tc2.data(), sizeof(int32_t) * u_tc2.size());
+    put(o_u_fuse_tc, u_fuse_tc.data(), sizeof(int32_t) * u_fuse_tc.size());
   }
 
   Tables tables(uint8_t* ws) const {
@@ -228,6 +235,7 @@ struct Layout {
     t.row0_out = reinterpret_cast<const int64_t*>(ws + o_row0);
     t.unit0_tc1 = reinterpret_cast<const int32_t*>(ws + o_u_tc1);
     t.unit0_tc2 = reinterpret_cast<const int32_t*>(ws + o_u_tc2);
+    t.unit0_fuse_tc = reinterpret_cast<const int32_t*>(ws + o_u_fuse_tc);
     t.status = reinterpret_cast<int32_t*>(ws + o_status);
     return t;
   }
@@ -257,6 +265,15 @@ cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, 
                            lse, row_lse, scores, st);
   return launch_score_simt(dtype, Qw, K, sh, tb, lay.units_lse, lay.units_col, lse, row_lse,
                            scores, st);
+}
+
+// Eq. (redistribution, weight_fusion) on tensor cores (bf16, d = 128) or CUDA cores.
+cudaError_t launch_fuse(int dtype, const void* V, const Layout& lay, const Shape& sh,
+                        const Tables& tb, const int32_t* keep, const int32_t* drop, float mu,
+                        float tau, void* V_out, cudaStream_t st) {
+  if (g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128)
+    return launch_fuse_tc(V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse_tc, st);
+  return launch_fuse_simt(dtype, V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse, st);
 }
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -433,7 +450,7 @@ int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int
   const Tables tb = lay.tables(w);
   e = launch_gather_k(dtype, K, sh, tb, keep_idx, K_out, lay.out_rows, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_fuse_simt(dtype, V, sh, tb, keep_idx, drop_idx, mu, tau, V_out, lay.units_fuse, st);
+  e = launch_fuse(dtype, V, lay, sh, tb, keep_idx, drop_idx, mu, tau, V_out, st);
   return cuda_status(e);
 }
 
@@ -471,7 +488,7 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   if (e != cudaSuccess) return VC_ERR_CUDA;
   e = launch_gather_k(p->dtype, K, sh, tb, idx_out, K_out, lay.out_rows, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_fuse_simt(p->dtype, V, sh, tb, idx_out, drop, p->mu, p->tau, V_out, lay.units_fuse, st);
+  e = launch_fuse(p->dtype, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, V_out, st);
   return cuda_status(e);
 }
 

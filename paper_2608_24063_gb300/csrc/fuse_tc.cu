@@ -1,0 +1,348 @@
+// Value fusion on the tcgen05 tensor cores, Eq. (redistribution) and
+// Eq. (weight_fusion); bf16 inputs, d = 128.
+//
+// One CTA per (request, layer, KV head, tile of 128 kept rows):
+//   O = softmax_row(V_k V_d^T / tau) V_d, online over tiles of 128 dropped rows,
+//   V_out = mu V_k + (1 - mu) O.
+// Kept and dropped rows are gathered by index with cp.async into 128-byte
+// swizzled tiles (the layout TMA would write).  S = V_k V_d^T and
+// O += P V_d run on tcgen05.mma with fp32 accumulators in tensor memory:
+// V_d is read K-major for the first product and MN-major for the second;
+// P goes through shared memory in bf16.  The softmax keeps a per-row
+// reference maximum and only rescales O (in tensor memory) when a tile's
+// maximum exceeds it by more than 2^8, so rescaling is rare.
+//
+// Warp roles (256 threads, one CTA per SM): warp 0 allocates tensor memory
+// and one of its threads issues the MMAs; warps 1-3 gather rows; warps 4-7
+// own one kept row each (= TMEM lane) for the softmax and the epilogue.
+// Every wait is bounded (see tc_common.cuh).
+#include "kernels.h"
+#include "profile.h"
+#include "tc_common.cuh"
+#include "vc_common.cuh"
+
+namespace vc {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 256;
+constexpr int kProducers = 96;                   // warps 1-3
+constexpr uint32_t kTile = 128;
+constexpr uint32_t kKB = kTile * 128;            // one K-block: 128 rows x 128 bytes
+constexpr int kVdStages = 3;
+constexpr uint32_t kTmemCols = 512;              // O: 0..127, S: 128..383
+constexpr float kRescaleLog2 = 8.f;
+
+struct FSmem {
+  uint8_t vk[2][kKB];                 // kept rows: A operand of S = V_k V_d^T
+  uint8_t vd[kVdStages][2][kKB];      // dropped rows: B operand of both products
+  uint8_t p[2][2][kKB];               // softmax numerators (bf16): A operand of O += P V_d
+  uint64_t vk_full;
+  uint64_t vd_full[kVdStages], vd_empty[kVdStages];
+  uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
+  uint64_t o_full, mma_done;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  const uint32_t a = smem_u32(p);
+  return p + ((1024u - (a & 1023u)) & 1023u);
+}
+
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  int dummy = 0;
+  mbar_wait(bar, parity, &dummy);
+}
+
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
+// Byte offset of 16-byte chunk c (0..15) of row r in a swizzled 128-row tile pair.
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return (uint32_t)((c >> 3) * kKB + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+}
+
+// Gather `count` rows (positions idx[0..count)) of a [n][128] bf16 slab into a
+// swizzled tile pair; rows >= count and bad positions are zero-filled.
+__device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* slab,
+                                            const int32_t* idx, int count, int n, int tid,
+                                            int32_t* status) {
+  for (int e = tid; e < (int)kTile * 16; e += kProducers) {
+    const int r = e >> 4, c = e & 15;
+    const __nv_bfloat16* src = slab;
+    uint32_t bytes = 0;
+    if (r < count) {
+      const int v = idx[r];
+      if (v >= 0 && v < n) {
+        src = slab + (int64_t)v * 128 + c * 8;
+        bytes = 16;
+      } else if (c == 0) {
+        set_status(status, VC_ERR_DEVICE_INDEX);
+      }
+    }
+    cp_async16(dst + swz(r, c), src, bytes);
+  }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
+                 const int32_t* __restrict__ keep_idx, const int32_t* __restrict__ drop_idx,
+                 float mu, float c2, __nv_bfloat16* __restrict__ V_out) {
+  extern __shared__ uint8_t smem_raw[];
+  FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)blockIdx.x);
+  const int r = rl / sh.L, l = rl % sh.L;
+  const Req rq = tb.req[r];
+  const Layer ly = tb.layer[rl];
+  const int ktiles = (ly.B + (int)kTile - 1) / (int)kTile;
+  const int u = blockIdx.x - tb.unit0_fuse_tc[rl];
+  const int g = u / ktiles;
+  const int r0 = (u % ktiles) * (int)kTile;
+  const int rows = min((int)kTile, ly.B - r0);
+  const int D = ly.D;
+  const int nt = (D + (int)kTile - 1) / (int)kTile;
+
+  const __nv_bfloat16* Vl = V + rq.kv_off + ((int64_t)l * sh.Hkv + g) * rq.n * 128;
+  const int64_t orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
+  const int32_t* kp = keep_idx + orow;
+  const int32_t* dp = drop_idx + rq.drop_row0 + (int64_t)sh.Hkv * ly.Qd + (int64_t)g * D;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&sm.vk_full, kProducers);
+    for (int i = 0; i < kVdStages; ++i) { mbar_init(&sm.vd_full[i], kProducers); mbar_init(&sm.vd_empty[i], 1); }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.s_full[i], 1);
+      mbar_init(&sm.s_empty[i], kTile);
+      mbar_init(&sm.p_full[i], kTile);
+      mbar_init(&sm.p_empty[i], 1);
+    }
+    mbar_init(&sm.o_full, 1);
+    mbar_init(&sm.mma_done, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = sm.tmem_base;
+  volatile int* abort = &sm.abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- MMA issuer
+      const uint32_t id_s = idesc_bf16_f32(kTile, kTile);
+      const uint32_t id_o = idesc_bf16_f32_bmn(kTile, kTile);
+      bool ok = mbar_wait(&sm.vk_full, 0, abort);
+      for (int j = 0; ok && j <= nt; ++j) {
+        if (j < nt) {
+          const int st = j % kVdStages, sb = j & 1;
+          if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
+          if (!mbar_wait(&sm.s_empty[sb], ((j >> 1) & 1) ^ 1, abort)) break;
+          tc_fence_after();
+          const uint32_t d = tbase + kTile + (uint32_t)sb * kTile;
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16(d, desc_sw128(smem_u32(sm.vk[kk >> 2]) + (kk & 3) * 32),
+                     desc_sw128(smem_u32(sm.vd[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
+          mma_commit(&sm.s_full[sb]);
+        }
+        if (j >= 1) {
+          const int jp = j - 1, pb = jp & 1, st = jp % kVdStages;
+          if (!mbar_wait(&sm.p_full[pb], (jp >> 1) & 1, abort)) break;
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16(tbase, desc_sw128(smem_u32(sm.p[pb][kk >> 2]) + (kk & 3) * 32),
+                     desc_sw128_mn(smem_u32(sm.vd[st][0]) + kk * 2048, kKB), id_o,
+                     (jp > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(&sm.p_empty[pb]);
+          mma_commit(&sm.vd_empty[st]);
+        }
+      }
+      mma_commit(&sm.o_full);
+      mma_commit(&sm.mma_done);
+      drain_wait(&sm.mma_done, 0);
+    }
+  } else if (warp < 4) {
+    // ---- row gathers (cp.async); a stage is published once its copies landed
+    const int tid = threadIdx.x - 32;
+    gather_tile(&sm.vk[0][0], Vl, kp, rows, rq.n, tid, tb.status);
+    cp_async_commit();
+    cp_async_wait<0>();
+    fence_proxy_async();
+    mbar_arrive(&sm.vk_full);
+    int j = 0;
+    for (; j < nt; ++j) {
+      const int st = j % kVdStages;
+      if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
+      gather_tile(&sm.vd[st][0][0], Vl, dp + j * (int)kTile, min((int)kTile, D - j * (int)kTile),
+                  rq.n, tid, tb.status);
+      cp_async_commit();
+      if (j >= 1) {
+        cp_async_wait<1>();
+        fence_proxy_async();
+        mbar_arrive(&sm.vd_full[(j - 1) % kVdStages]);
+      }
+    }
+    cp_async_wait<0>();
+    fence_proxy_async();
+    if (j >= 1) mbar_arrive(&sm.vd_full[(j - 1) % kVdStages]);
+  } else {
+    // ---- softmax over the drop set and epilogue: one thread per kept row
+    const int row = threadIdx.x - 128;
+    const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    float m = -INFINITY, lsum = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt; ++j) {
+      const int sb = j & 1;
+      if (!warp_wait(&sm.s_full[sb], (j >> 1) & 1, abort)) { ok = false; break; }
+      tc_fence_after();
+      float x[8][16];
+#pragma unroll
+      for (int p = 0; p < 8; ++p) {
+        uint32_t v[16];
+        tmem_ld16(tbase + lane_off + kTile + sb * kTile + p * 16, v);
+        tmem_wait(v);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[q]);
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.s_empty[sb]);
+      const int valid = min((int)kTile, D - j * (int)kTile);
+      float tm = -INFINITY;
+#pragma unroll
+      for (int p = 0; p < 8; ++p)
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          if (p * 16 + q >= valid) x[p][q] = -INFINITY;
+          tm = fmaxf(tm, x[p][q]);
+        }
+      tm *= c2;
+      // raise the reference maximum when this tile exceeds it by more than 2^8
+      const bool raise = tm > m + kRescaleLog2;
+      const float m_new = raise ? tm : m;
+      const float corr = raise ? exp2f(m - m_new) : 1.f;   // 0 on the first tile
+      if (__any_sync(0xffffffffu, raise && j > 0)) {
+        // O holds the tiles before j: wait for their last product, then rescale in place
+        if (!warp_wait(&sm.p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll 1
+        for (int p = 0; p < 8; ++p) {
+          uint32_t v[16];
+          tmem_ld16(tbase + lane_off + p * 16, v);
+          tmem_wait(v);
+#pragma unroll
+          for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
+          tmem_st16(tbase + lane_off + p * 16, v);
+        }
+        tmem_wait_st();
+      }
+      lsum *= corr;
+      m = m_new;
+      // numerators in bf16 into the P tile (row-major, swizzled, K-major A operand)
+      if (!warp_wait(&sm.p_empty[sb], ((j >> 1) & 1) ^ 1, abort)) { ok = false; break; }
+      uint8_t* pt = &sm.p[sb][0][0];
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        float e[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          e[q] = exp2f(fmaf(x[c >> 1][(c & 1) * 8 + q], c2, -m));
+          lsum += e[q];
+        }
+        uint4 w;
+        w.x = pack_bf16x2(e[0], e[1]);
+        w.y = pack_bf16x2(e[2], e[3]);
+        w.z = pack_bf16x2(e[4], e[5]);
+        w.w = pack_bf16x2(e[6], e[7]);
+        *reinterpret_cast<uint4*>(pt + swz(row, c)) = w;
+      }
+      fence_proxy_async();
+      tc_fence_before();
+      mbar_arrive(&sm.p_full[sb]);
+    }
+    // epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped;
+    // the kept rows are read from shared memory once their gather has landed
+    const bool have_k = warp_wait(&sm.vk_full, 0, abort);
+    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
+    if (have_o) tc_fence_after();
+    const float w_o = have_o ? (1.f - mu) / lsum : 0.f;
+    const float w_k = have_o ? mu : 1.f;
+#pragma unroll 1
+    for (int p = 0; p < 8; ++p) {
+      float o[16];
+      if (have_o) {
+        uint32_t v[16];
+        tmem_ld16(tbase + lane_off + p * 16, v);
+        tmem_wait(v);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) o[q] = __uint_as_float(v[q]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 16; ++q) o[q] = 0.f;
+      }
+      if (have_k && row < rows) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int c = p * 2 + h;
+          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[0][0] + swz(row, c));
+          const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
+          uint4 w;
+          uint32_t* wp = &w.x;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float2 kf = __bfloat1622float2(k2[q]);
+            const float a = fmaf(w_k, kf.x, w_o * o[h * 8 + 2 * q]);
+            const float b = fmaf(w_k, kf.y, w_o * o[h * 8 + 2 * q + 1]);
+            wp[q] = pack_bf16x2(a, b);
+          }
+          *reinterpret_cast<uint4*>(V_out + (orow + row) * 128 + c * 8) = w;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+  if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+}
+
+}  // namespace
+
+int fuse_rows_per_tile_tc() { return (int)kTile; }
+
+cudaError_t launch_fuse_tc(const void* V, const Shape& sh, const Tables& tb,
+                           const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
+                           void* V_out, int units, cudaStream_t st) {
+  if (units == 0) return cudaSuccess;
+  const size_t smem = sizeof(FSmem) + 1024;
+  cudaError_t e = cudaFuncSetAttribute(fuse_v_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  ProfileScope ps("fuse_v_tc", st);
+  fuse_v_tc_kernel<<<units, kThreads, smem, st>>>(
+      static_cast<const __nv_bfloat16*>(V), sh, tb, keep_idx, drop_idx, mu, kLog2e / tau,
+      static_cast<__nv_bfloat16*>(V_out));
+  return cudaGetLastError();
+}
+
+}  // namespace vc

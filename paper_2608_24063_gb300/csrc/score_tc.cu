@@ -239,6 +239,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
+    __syncwarp();
     tc_fence_after();
     tmem_dealloc(tbase, kTmemCols);
   }
@@ -463,6 +464,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
+    __syncwarp();
     tc_fence_after();
     tmem_dealloc(tbase, kTmemCols);
   }

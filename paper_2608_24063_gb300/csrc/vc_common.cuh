@@ -50,6 +50,7 @@ struct Tables {              // device pointers into the workspace
   const int64_t* row0_out;   // [n_req * L + 1] first output row of each (request, layer)
   const int32_t* unit0_tc1;  // [n_req + 1] CTAs of the tensor-core lse pass
   const int32_t* unit0_tc2;  // [n_req + 1] CTAs of the tensor-core column-sum pass
+  const int32_t* unit0_fuse_tc;  // [n_req * L + 1] 128-row kept tiles x Hkv (tensor-core fusion)
   int32_t* status;           // device status word
 };
 

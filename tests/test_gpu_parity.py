@@ -192,6 +192,48 @@ def test_tensor_core_scores_match_oracle_and_cuda_cores(shape, mode):
         assert float(err.max()) < 2e-5, float(err.max())
 
 
+FUSE_CASES = [
+    # n, B, D, mu, tau
+    (300, 1, 1, 0.7, 1.0),
+    (300, 129, 127, 0.7, 1.0),
+    (600, 128, 129, 0.0, 0.5),
+    (1000, 300, 500, 0.7, 4.0),
+    (2000, 257, 1500, 0.3, 1.0),
+    (500, 200, 0, 0.7, 1.0),
+    (700, 130, 260, 1.0, 1.0),
+]
+
+
+@pytest.mark.parametrize("case", FUSE_CASES)
+def test_tensor_core_fusion_matches_oracle(case, kernel_path):
+    n, b, D, mu, tau = case
+    L, Hkv, d = 1, 2, 128
+    K = _rand((L, Hkv, n, d), 7000 + n + b, torch.bfloat16)
+    V = _rand((L, Hkv, n, d), 7100 + n + D, torch.bfloat16)
+    rng = np.random.default_rng(n * 7 + b)
+    keep, drop = [], []
+    for g in range(Hkv):
+        perm = rng.permutation(n)
+        keep.append(np.sort(perm[:b]))
+        drop.append(np.sort(perm[b:b + D]))
+    keep_t = torch.tensor(np.concatenate(keep), dtype=torch.int32, device=DEV)
+    drop_t = torch.tensor(np.concatenate(drop), dtype=torch.int32, device=DEV)
+    Ko, Vo = vc.prunekv_fuse_compact(K.to(DEV), V.to(DEV), [b], b + D, keep_t, drop_t, mu, tau)
+    torch.cuda.synchronize()
+    Vn = np64(V)
+    got = np64(Vo)
+    for g in range(Hkv):
+        ref = ok.fuse_values(Vn[0, g], keep[g], drop[g], mu, tau)
+        sl = got[g * b:(g + 1) * b]
+        diff = np.abs(sl - ref)
+        rms = float(np.sqrt((ref ** 2).mean()))
+        assert float(diff.max()) <= 2e-2 * float(np.abs(ref).max())
+        assert not (diff > 2e-2 * np.abs(ref) + 2e-2 * rms).any()
+        if mu == 1.0 or D == 0:
+            assert np.array_equal(sl, Vn[0, g][keep[g]])
+        assert torch.equal(Ko[g * b:(g + 1) * b].cpu(), K[0, g][torch.from_numpy(keep[g])])
+
+
 # ---------------------------------------------------------------------------
 # The workloads at full size.
 

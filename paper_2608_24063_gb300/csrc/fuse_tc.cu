@@ -38,12 +38,14 @@ struct FSmem {
   uint8_t vk[2][kKB];                 // kept rows: A operand of S = V_k V_d^T
   uint8_t vd[kVdStages][2][kKB];      // dropped rows: B operand of both products
   uint8_t p[2][2][kKB];               // softmax numerators (bf16): A operand of O += P V_d
+  int32_t idx[1 + kVdStages][kTile];  // row positions of the kept tile and of each drop stage
   uint64_t vk_full;
   uint64_t vd_full[kVdStages], vd_empty[kVdStages];
   uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
   uint64_t o_full, mma_done;
   uint32_t tmem_base;
   int abort;
+  int gather_go;
 };
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -66,25 +68,27 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
   return (uint32_t)((c >> 3) * kKB + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
 
-// Gather `count` rows (positions idx[0..count)) of a [n][128] bf16 slab into a
-// swizzled tile pair; rows >= count and bad positions are zero-filled.
-__device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* slab,
-                                            const int32_t* idx, int count, int n, int tid,
+// Row position r of a tile whose positions are pos[0..count): -1 (zero row)
+// beyond count or for a position outside [0, n) (recorded in the status word).
+__device__ __forceinline__ int32_t tile_pos(const int32_t* pos, int count, int r, int n,
                                             int32_t* status) {
+  if (r >= count) return -1;
+  const int32_t v = pos[r];
+  if (v < 0 || v >= n) {
+    set_status(status, VC_ERR_DEVICE_INDEX);
+    return -1;
+  }
+  return v;
+}
+
+// Gather the 128 rows listed in idx (shared memory, -1 = zeros) of a [n][128]
+// bf16 slab into a swizzled tile pair; 16 consecutive threads copy one row.
+__device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* slab,
+                                            const int32_t* idx, int tid) {
   for (int e = tid; e < (int)kTile * 16; e += kProducers) {
     const int r = e >> 4, c = e & 15;
-    const __nv_bfloat16* src = slab;
-    uint32_t bytes = 0;
-    if (r < count) {
-      const int v = idx[r];
-      if (v >= 0 && v < n) {
-        src = slab + (int64_t)v * 128 + c * 8;
-        bytes = 16;
-      } else if (c == 0) {
-        set_status(status, VC_ERR_DEVICE_INDEX);
-      }
-    }
-    cp_async16(dst + swz(r, c), src, bytes);
+    const int32_t v = idx[r];
+    cp_async16(dst + swz(r, c), v >= 0 ? slab + (int64_t)v * 128 + c * 8 : slab, v >= 0 ? 16u : 0u);
   }
 }
 
@@ -179,19 +183,37 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
       drain_wait(&sm.mma_done, 0);
     }
   } else if (warp < 4) {
-    // ---- row gathers (cp.async); a stage is published once its copies landed
+    // ---- row gathers (cp.async).  The positions of a tile go to shared memory
+    // first (fetched one tile ahead), so the copies issue back to back; a
+    // stage is published once its copies landed.
     const int tid = threadIdx.x - 32;
-    gather_tile(&sm.vk[0][0], Vl, kp, rows, rq.n, tid, tb.status);
+    sm.idx[0][tid] = tile_pos(kp, rows, tid, rq.n, tb.status);
+    if (tid + kProducers < (int)kTile) sm.idx[0][tid + kProducers] = tile_pos(kp, rows, tid + kProducers, rq.n, tb.status);
+    named_sync(1, kProducers);
+    gather_tile(&sm.vk[0][0], Vl, sm.idx[0], tid);
     cp_async_commit();
     cp_async_wait<0>();
     fence_proxy_async();
     mbar_arrive(&sm.vk_full);
+    int cnt = min((int)kTile, D);
+    int32_t a0 = nt > 0 ? tile_pos(dp, cnt, tid, rq.n, tb.status) : -1;
+    int32_t a1 = nt > 0 && tid + kProducers < (int)kTile ? tile_pos(dp, cnt, tid + kProducers, rq.n, tb.status) : -1;
     int j = 0;
     for (; j < nt; ++j) {
       const int st = j % kVdStages;
-      if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
-      gather_tile(&sm.vd[st][0][0], Vl, dp + j * (int)kTile, min((int)kTile, D - j * (int)kTile),
-                  rq.n, tid, tb.status);
+      int32_t* buf = sm.idx[1 + st];
+      buf[tid] = a0;
+      if (tid + kProducers < (int)kTile) buf[tid + kProducers] = a1;
+      if (tid == 0) sm.gather_go = mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort) ? 1 : 0;
+      named_sync(1, kProducers);
+      if (!sm.gather_go) break;
+      if (j + 1 < nt) {
+        const int32_t* nxt = dp + (j + 1) * (int)kTile;
+        cnt = min((int)kTile, D - (j + 1) * (int)kTile);
+        a0 = tile_pos(nxt, cnt, tid, rq.n, tb.status);
+        a1 = tid + kProducers < (int)kTile ? tile_pos(nxt, cnt, tid + kProducers, rq.n, tb.status) : -1;
+      }
+      gather_tile(&sm.vd[st][0][0], Vl, buf, tid);
       cp_async_commit();
       if (j >= 1) {
         cp_async_wait<1>();
@@ -213,13 +235,17 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
       if (!warp_wait(&sm.s_full[sb], (j >> 1) & 1, abort)) { ok = false; break; }
       tc_fence_after();
       float x[8][16];
+      {
+        uint32_t v[8][16];
 #pragma unroll
-      for (int p = 0; p < 8; ++p) {
-        uint32_t v[16];
-        tmem_ld16(tbase + lane_off + kTile + sb * kTile + p * 16, v);
-        tmem_wait(v);
+        for (int p = 0; p < 8; ++p) tmem_ld16(tbase + lane_off + kTile + sb * kTile + p * 16, v[p]);
+        tmem_wait_only();
 #pragma unroll
-        for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[q]);
+        for (int p = 0; p < 8; ++p) {
+          reg_fence(v[p]);
+#pragma unroll
+          for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
+        }
       }
       tc_fence_before();
       mbar_arrive(&sm.s_empty[sb]);
@@ -236,19 +262,24 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
       // raise the reference maximum when this tile exceeds it by more than 2^8
       const bool raise = tm > m + kRescaleLog2;
       const float m_new = raise ? tm : m;
-      const float corr = raise ? exp2f(m - m_new) : 1.f;   // 0 on the first tile
+      const float corr = raise ? ex2(m - m_new) : 1.f;     // 0 on the first tile
       if (__any_sync(0xffffffffu, raise && j > 0)) {
         // O holds the tiles before j: wait for their last product, then rescale in place
         if (!warp_wait(&sm.p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll 1
-        for (int p = 0; p < 8; ++p) {
-          uint32_t v[16];
-          tmem_ld16(tbase + lane_off + p * 16, v);
-          tmem_wait(v);
+        for (int h = 0; h < 2; ++h) {
+          uint32_t v[4][16];
 #pragma unroll
-          for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
-          tmem_st16(tbase + lane_off + p * 16, v);
+          for (int p = 0; p < 4; ++p) tmem_ld16(tbase + lane_off + (h * 4 + p) * 16, v[p]);
+          tmem_wait_only();
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            reg_fence(v[p]);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) v[p][q] = __float_as_uint(__uint_as_float(v[p][q]) * corr);
+            tmem_st16(tbase + lane_off + (h * 4 + p) * 16, v[p]);
+          }
         }
         tmem_wait_st();
       }
@@ -262,7 +293,7 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
         float e[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          e[q] = exp2f(fmaf(x[c >> 1][(c & 1) * 8 + q], c2, -m));
+          e[q] = ex2(fmaf(x[c >> 1][(c & 1) * 8 + q], c2, -m));
           lsum += e[q];
         }
         uint4 w;
@@ -283,19 +314,24 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
     if (have_o) tc_fence_after();
     const float w_o = have_o ? (1.f - mu) / lsum : 0.f;
     const float w_k = have_o ? mu : 1.f;
-#pragma unroll 1
+    uint32_t ov[8][16];
+    if (have_o) {
+#pragma unroll
+      for (int p = 0; p < 8; ++p) tmem_ld16(tbase + lane_off + p * 16, ov[p]);
+      tmem_wait_only();
+#pragma unroll
+      for (int p = 0; p < 8; ++p) reg_fence(ov[p]);
+    } else {
+#pragma unroll
+      for (int p = 0; p < 8; ++p)
+#pragma unroll
+        for (int q = 0; q < 16; ++q) ov[p][q] = 0u;
+    }
+#pragma unroll
     for (int p = 0; p < 8; ++p) {
       float o[16];
-      if (have_o) {
-        uint32_t v[16];
-        tmem_ld16(tbase + lane_off + p * 16, v);
-        tmem_wait(v);
 #pragma unroll
-        for (int q = 0; q < 16; ++q) o[q] = __uint_as_float(v[q]);
-      } else {
-#pragma unroll
-        for (int q = 0; q < 16; ++q) o[q] = 0.f;
-      }
+      for (int q = 0; q < 16; ++q) o[q] = __uint_as_float(ov[p][q]);
       if (have_k && row < rows) {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {

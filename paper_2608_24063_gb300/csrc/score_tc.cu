@@ -60,15 +60,6 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, ok);
 }
 
-// 16 consecutive TMEM columns of this thread's lane, as floats.
-__device__ __forceinline__ void tmem_cols16(uint32_t taddr, float (&x)[16]) {
-  uint32_t r[16];
-  tmem_ld16(taddr, r);
-  tmem_wait(r);
-#pragma unroll
-  for (int j = 0; j < 16; ++j) x[j] = __uint_as_float(r[j]);
-}
-
 __device__ __forceinline__ float sum16(const float (&e)[16]) {
   float a[8];
 #pragma unroll
@@ -200,8 +191,18 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {            // two halves of 64 columns
         float x[4][16];
+        {
+          uint32_t v[4][16];
 #pragma unroll
-        for (int p = 0; p < 4; ++p) tmem_cols16(col0 + h * 64 + p * 16, x[p]);
+          for (int p = 0; p < 4; ++p) tmem_ld16(col0 + h * 64 + p * 16, v[p]);
+          tmem_wait_only();
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            reg_fence(v[p]);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
+          }
+        }
         if (h == 1) {
           tc_fence_before();
           mbar_arrive(&sm.tm_empty[b][slot]);   // columns copied out: the MMA may reuse them
@@ -216,7 +217,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           }
         const float xm = cm * s2;
         if (xm > m) {
-          const float c = exp2f(m - xm);
+          const float c = ex2(m - xm);
           z.s *= c;
           z.c *= c;
           m = xm;
@@ -226,7 +227,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           for (int p = 0; p < 4; ++p) {
             float e[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) e[j] = exp2f(fmaf(x[p][j], s2, -m));
+            for (int j = 0; j < 16; ++j) e[j] = ex2(fmaf(x[p][j], s2, -m));
             z.add(sum16(e));
           }
         }
@@ -422,9 +423,20 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
           for (int p0 = 0; p0 < ncol; p0 += 64) {
             const int np = min(4, (ncol - p0) >> 4);
             float x[4][16];
+            {
+              uint32_t v[4][16];
 #pragma unroll
-            for (int p = 0; p < 4; ++p)
-              if (p < np) tmem_cols16(col0 + p0 + p * 16, x[p]);
+              for (int p = 0; p < 4; ++p)
+                if (p < np) tmem_ld16(col0 + p0 + p * 16, v[p]);
+              tmem_wait_only();
+#pragma unroll
+              for (int p = 0; p < 4; ++p)
+                if (p < np) {
+                  reg_fence(v[p]);
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
+                }
+            }
             if (p0 + 64 >= ncol) {
               tc_fence_before();
               mbar_arrive(&sm.tm_empty[qs]);
@@ -434,7 +446,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
               if (p < np) {
                 float e[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) e[j] = exp2f(fmaf(x[p][j], s2, -buf[p0 + p * 16 + j]));
+                for (int j = 0; j < 16; ++j) e[j] = ex2(fmaf(x[p][j], s2, -buf[p0 + p * 16 + j]));
                 lay.add(sum16(e));
               }
             }

@@ -125,7 +125,7 @@ int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t H
  * fixed device array of VC_STATIC_SCRATCH_BYTES inside the library, which
  * every GPU that loads the library holds until the process exits.
  *   - Problems needing more scratch than that (prunekv_score_workspace_size
- *     (L, Hq, W) > VC_STATIC_SCRATCH_BYTES, i.e. roughly L*Hq*W > 1,000,000
+ *     (L, Hq, W) > VC_STATIC_SCRATCH_BYTES, i.e. roughly L*Hq*W > 800,000
  *     window rows) are rejected with VC_ERR_WORKSPACE before any device work.
  *   - The first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress) with that device current and caches it; make
@@ -136,7 +136,7 @@ int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t H
  *   - Device-side status is kept in the shared array and is not reported;
  *     the return value covers arguments and launches.
  */
-#define VC_STATIC_SCRATCH_BYTES (4u << 20)
+#define VC_STATIC_SCRATCH_BYTES (16u << 20)
 int prunekv_score_static(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq,
                          int32_t Hkv, int32_t d, int32_t n_vis, int32_t W, float scale,
                          int rank_mode, const float* row_lse, float* scores, void* stream);

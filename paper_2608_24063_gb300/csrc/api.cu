@@ -52,7 +52,7 @@ struct Layout {
   bool need_lse = false, need_scores = false, need_sort = false, need_drop = false;
   // tensor-core score plan
   int S = 1;
-  int64_t q_rows = 0, k_rows = 0, max_rows = 0;
+  int64_t q_rows = 0, k_rows = 0, max_rows = 0, prows = 0, max_prows = 0;
   std::vector<int32_t> u_tc1, u_tc2, base_tc1, u_fuse_tc;
   int units_fuse_tc = 0;
   // derived sizes
@@ -61,7 +61,7 @@ struct Layout {
   // workspace offsets
   size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
          o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, o_u_fuse_tc = 0, table_begin = 0, table_end = 0, o_lse = 0,
-         o_part = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
+         o_part = 0, o_lsep = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
   // host images
   std::vector<Req> req;
   std::vector<Layer> layer;
@@ -81,7 +81,7 @@ struct Layout {
     u_fuse_tc.assign((size_t)n_req * L + 1, 0);
     u_tc2.assign(n_req + 1, 0);
     base_tc1.assign(n_req, 0);
-    q_rows = k_rows = max_rows = 0;
+    q_rows = k_rows = max_rows = prows = max_prows = 0;
     int64_t cu_n = 0, cu_w = 0;
     const int per_req_problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
     const int rows_tile = score_rows_per_tile_simt(), keys_tile = score_keys_per_tile_simt();
@@ -98,6 +98,9 @@ struct Layout {
       q.drop_row0 = drop_rows;
       q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
       q.C = (G * p.W + 127) / 128;
+      q.lsep_off = prows;
+      prows += (int64_t)L * Hkv * q.C * 128;
+      max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
       q.nrb = (G * p.W + 255) / 256;
       q.tiles = (p.n + 127) / 128;
       base_tc1[r] = L * Hkv * q.nrb;
@@ -147,8 +150,10 @@ struct Layout {
     o_u_fuse_tc = a.take(sizeof(int32_t) * u_fuse_tc.size());
     table_end = a.off;
     if (need_lse) {
-      o_lse = a.take(sizeof(float) * lse_elems);
-      o_part = a.take(sizeof(float2) * lse_elems * score_tc_max_splits());
+      // CUDA-core path: lse rows; tensor-core path: split partials (same region)
+      // and the chunk-padded normalisers
+      o_lse = o_part = a.take(sizeof(float2) * lse_elems * score_tc_max_splits());
+      o_lsep = a.take(sizeof(float) * prows);
     }
     if (need_scores) o_scores = a.take(sizeof(float) * score_elems);
     if (need_sort) {
@@ -187,6 +192,7 @@ struct Layout {
     t.q_rows = q_rows;
     t.k_rows = k_rows;
     t.max_rows = max_rows;
+    t.max_prows = max_prows;
     return t;
   }
 
@@ -262,7 +268,7 @@ cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, 
   float* lse = reinterpret_cast<float*>(w + lay.o_lse);
   if (tc)
     return launch_score_tc(Qw, K, sh, tb, lay.tc_plan(), reinterpret_cast<float2*>(w + lay.o_part),
-                           lse, row_lse, scores, st);
+                           reinterpret_cast<float*>(w + lay.o_lsep), row_lse, scores, st);
   return launch_score_simt(dtype, Qw, K, sh, tb, lay.units_lse, lay.units_col, lse, row_lse,
                            scores, st);
 }
@@ -376,7 +382,8 @@ int viscache_set_kernel_path(int path) {
 
 size_t prunekv_score_workspace_size(int32_t L, int32_t Hq, int32_t W) {
   if (L < 1 || L > 256 || Hq < 1 || W < 1) return 0;
-  return score_layout(L, Hq, 1, 64, 1, W, VC_RANK_SHARED).total;
+  // Hkv = Hq bounds the chunk padding of any Hkv dividing Hq
+  return score_layout(L, Hq, Hq, 128, 1, W, VC_RANK_SHARED).total;
 }
 
 int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq, int32_t Hkv,

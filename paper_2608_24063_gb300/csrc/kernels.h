@@ -32,10 +32,11 @@ struct TcPlan {
   int64_t q_rows;    // rows of the packed Qw tensor
   int64_t k_rows;    // rows of the packed K tensor
   int64_t max_rows;  // max over requests of L*Hq*W
+  int64_t max_prows; // max over requests of L*Hkv*C*128 (chunk-padded rows)
 };
 int score_tc_max_splits();
 cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
-                            const TcPlan& tp, float2* part, float* lse2, const float* lse_nat,
+                            const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
                             float* scores, cudaStream_t st);
 
 // V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on tcgen05 tensor cores (bf16, d = 128).

@@ -9,15 +9,21 @@
 //   pass 1 (score_lse_tc)    rows in TMEM lanes: per row, running max and
 //                            compensated sum of exp2 over a range of key
 //                            tiles -> partial (m, z) per key split;
-//   merge  (lse_merge)       lse2 = m + log2 z over the splits (or the
-//                            caller's natural-log normaliser * log2 e);
+//   merge  (lse_merge)       -lse2 = -(m + log2 z) over the splits (or minus
+//                            the caller's natural-log normaliser * log2 e),
+//                            written per (layer, KV head) in 128-row chunks
+//                            padded with -inf;
 //   pass 2 (score_colsum_tc) keys in TMEM lanes: each thread owns one key and
 //                            sums exp2(x*scale*log2e - lse2[row]) over all
 //                            rows of all layers (compensated), s = sum / L.
+//                            The chunk's normalisers arrive with its Q rows
+//                            (one bulk copy), padding rows contribute 0.
 //
-// Warp roles in both passes (384 threads, one CTA per SM): warp 0 issues TMA,
-// warp 1 issues MMAs (one thread), warp 2 owns the tensor-memory allocation,
-// warps 4-7 and 8-11 are two consumer warpgroups.  Every wait is bounded: on a
+// Warp roles in both passes (320 threads, one CTA per SM): warps 0-3 and 4-7
+// are two consumer warpgroups (one TMEM lane per thread), warp 8 issues TMA and
+// owns the tensor-memory allocation, one thread of warp 9 issues the MMAs.
+// Each consumer thread takes a whole tile (up to 128 accumulators) per step,
+// so its exps and sums form many independent chains.  Every wait is bounded: on a
 // timeout the CTA stops issuing, waits for its own copies and MMAs, frees its
 // tensor memory and records VC_ERR_DEVICE_TIMEOUT.
 #include <cudaTypedefs.h>
@@ -34,7 +40,8 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 384;
+constexpr int kThreads = 320;
+constexpr int kProducerWarp = 8, kMmaWarp = 9;
 constexpr uint32_t kTile = 128;                 // keys per tile, rows per block / chunk
 constexpr uint32_t kKBlockBytes = kTile * 128;  // 128 rows x 64 bf16
 constexpr uint32_t kTileBytes = 2 * kKBlockBytes;
@@ -60,13 +67,21 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, ok);
 }
 
-__device__ __forceinline__ float sum16(const float (&e)[16]) {
-  float a[8];
+// sum_j exp2(x_j * s + b_j) over 16 values, with packed fp32x2 FMA and adds
+// (pairwise, so the rounding error stays a few ulp).
+__device__ __forceinline__ float exp2_sum16(const float (&x)[16], float2 s, const float2 (&b)[8]) {
+  float2 e[8];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) a[j] = e[2 * j] + e[2 * j + 1];
+  for (int j = 0; j < 8; ++j) {
+    const float2 t = __ffma2_rn(make_float2(x[2 * j], x[2 * j + 1]), s, b[j]);
+    e[j] = make_float2(ex2(t.x), ex2(t.y));
+  }
 #pragma unroll
-  for (int j = 0; j < 4; ++j) a[j] = a[2 * j] + a[2 * j + 1];
-  return (a[0] + a[1]) + (a[2] + a[3]);
+  for (int j = 0; j < 4; ++j) e[j] = __fadd2_rn(e[2 * j], e[2 * j + 1]);
+  e[0] = __fadd2_rn(e[0], e[1]);
+  e[2] = __fadd2_rn(e[2], e[3]);
+  e[0] = __fadd2_rn(e[0], e[2]);
+  return e[0].x + e[0].y;
 }
 
 // ---------------------------------------------------------------------------
@@ -115,7 +130,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (warp == 2) {
+  if (warp == kProducerWarp) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -125,7 +140,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
-  if (warp == 0 && lane == 0) {
+  if (warp == kProducerWarp && lane == 0) {
     // ---- TMA producer
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
@@ -146,7 +161,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     drain_wait(&sm.q_full, 0);
     for (int i = max(0, issued - kStages1); i < issued; ++i)
       drain_wait(&sm.k_full[i % kStages1], (i / kStages1) & 1);
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == kMmaWarp && lane == 0) {
     // ---- MMA issuer
     const uint32_t idesc = idesc_bf16_f32(kTile, kTile);
     bool ok = mbar_wait(&sm.q_full, 0, abort);
@@ -172,9 +187,9 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     }
     mma_commit(&sm.mma_done);
     drain_wait(&sm.mma_done, 0);
-  } else if (warp >= 4) {
+  } else if (warp < 8) {
     // ---- row statistics: one thread per row (= TMEM lane)
-    const int b = (warp - 4) >> 2;
+    const int b = warp >> 2;
     const int lrow = ((warp & 3) << 5) + lane;
     const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
     const float s2 = sh.scale_log2;
@@ -188,49 +203,52 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       tc_fence_after();
       const int valid = min((int)kTile, rq.n - (t_begin + i) * (int)kTile);
       const uint32_t col0 = tbase + lane_off + (uint32_t)(b * 2 + slot) * kTile;
-#pragma unroll 1
-      for (int h = 0; h < 2; ++h) {            // two halves of 64 columns
-        float x[4][16];
-        {
-          uint32_t v[4][16];
+      float x[8][16];
+      {
+        uint32_t v[8][16];
 #pragma unroll
-          for (int p = 0; p < 4; ++p) tmem_ld16(col0 + h * 64 + p * 16, v[p]);
-          tmem_wait_only();
+        for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, v[p]);
+        tmem_wait_only();
 #pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            reg_fence(v[p]);
+        for (int p = 0; p < 8; ++p) {
+          reg_fence(v[p]);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
-          }
+          for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
         }
-        if (h == 1) {
-          tc_fence_before();
-          mbar_arrive(&sm.tm_empty[b][slot]);   // columns copied out: the MMA may reuse them
-        }
-        float cm = -INFINITY;
+      }
+      tc_fence_before();
+      mbar_arrive(&sm.tm_empty[b][slot]);       // columns copied out: the MMA may reuse them
+      if (valid < (int)kTile) {                 // last tile of the request: mask keys >= n
 #pragma unroll
-        for (int p = 0; p < 4; ++p)
+        for (int p = 0; p < 8; ++p)
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            if (h * 64 + p * 16 + j >= valid) x[p][j] = -INFINITY;
-            cm = fmaxf(cm, x[p][j]);
-          }
-        const float xm = cm * s2;
-        if (xm > m) {
-          const float c = ex2(m - xm);
-          z.s *= c;
-          z.c *= c;
-          m = xm;
-        }
-        if (m != -INFINITY) {
+          for (int j = 0; j < 16; ++j)
+            if (p * 16 + j >= valid) x[p][j] = -INFINITY;
+      }
+      float pm[8];
 #pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            float e[16];
+      for (int p = 0; p < 8; ++p) {
+        float a = fmaxf(x[p][0], x[p][1]);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) e[j] = ex2(fmaf(x[p][j], s2, -m));
-            z.add(sum16(e));
-          }
-        }
+        for (int j = 2; j < 16; j += 2) a = fmax3(a, x[p][j], x[p][j + 1]);
+        pm[p] = a;
+      }
+      const float cm = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
+      const float xm = cm * s2;
+      if (xm > m) {
+        const float c = ex2(m - xm);
+        z.s *= c;
+        z.c *= c;
+        m = xm;
+      }
+      if (m != -INFINITY) {
+        float2 nb[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) nb[j] = make_float2(-m, -m);
+        float ps[8];
+#pragma unroll
+        for (int p = 0; p < 8; ++p) ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
+        z.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
       }
     }
     const int rho = rbp * 256 + b * (int)kTile + lrow;
@@ -239,7 +257,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) {
+  if (warp == kProducerWarp) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tbase, kTmemCols);
@@ -248,27 +266,36 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 }
 
 // ---------------------------------------------------------------------------
-// merge: lse2 per window row; grid (rows / 256, n_req)
+// merge: minus lse2 per window row into the chunk-padded layout; grid
+// (padded rows / 256, n_req)
 
 __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __restrict__ part,
-                                 const float* __restrict__ lse_nat, float* __restrict__ lse2) {
+                                 const float* __restrict__ lse_nat, float* __restrict__ nlse) {
   const Req rq = tb.req[blockIdx.y];
-  const int64_t per = (int64_t)sh.L * sh.Hq * rq.W;
+  const int cw = rq.C * (int)kTile;
+  const int64_t per = (int64_t)sh.L * sh.Hkv * cw;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= per) return;
-  const int64_t o = rq.lse_off + i;
-  if (lse_nat) {
-    lse2[o] = lse_nat[o] * kLog2e;
-    return;
+  const int p = (int)(i % cw);
+  const int grp = (int)(i / cw);
+  const int l = grp / sh.Hkv, g = grp % sh.Hkv;
+  float out = -INFINITY;                      // padding rows: exp2(x + -inf) = 0
+  if (p < sh.G * rq.W) {
+    const int64_t o = rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + p;
+    if (lse_nat) {
+      out = -lse_nat[o] * kLog2e;
+    } else {
+      float m = -INFINITY;
+      for (int s = 0; s < S; ++s) m = fmaxf(m, part[o * S + s].x);
+      float z = 0.f;
+      for (int s = 0; s < S; ++s) {
+        const float2 q = part[o * S + s];
+        if (q.x != -INFINITY) z += q.y * exp2f(q.x - m);
+      }
+      out = -(m + log2f(z));
+    }
   }
-  float m = -INFINITY;
-  for (int s = 0; s < S; ++s) m = fmaxf(m, part[o * S + s].x);
-  float z = 0.f;
-  for (int s = 0; s < S; ++s) {
-    const float2 p = part[o * S + s];
-    if (p.x != -INFINITY) z += p.y * exp2f(p.x - m);
-  }
-  lse2[o] = m + log2f(z);
+  nlse[rq.lsep_off + i] = out;
 }
 
 // ---------------------------------------------------------------------------
@@ -277,7 +304,7 @@ __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __res
 struct P2Smem {
   uint8_t k[2][2][kKBlockBytes];          // [stage = layer & 1][K-block]
   uint8_t q[kQStages][2][kKBlockBytes];   // [stage][K-block]
-  float lse[2][2][kTile];                 // [warpgroup][buffer][row]
+  float nlse[kQStages][kTile];            // minus lse2 of the stage's rows (-inf = padding)
   float red[2][kTile];                    // [warpgroup][key]
   uint64_t k_full[2], k_empty[2];
   uint64_t q_full[kQStages], q_empty[kQStages];
@@ -287,15 +314,10 @@ struct P2Smem {
   int abort;
 };
 
-// MMA columns of chunk c: the remaining rows rounded up to a multiple of 16.
-__device__ __forceinline__ int chunk_cols(int rows, int c) {
-  const int left = min((int)kTile, rows - c * (int)kTile);
-  return (left + 15) & ~15;
-}
 
 __global__ void __launch_bounds__(kThreads, 1)
 score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                       Shape sh, Tables tb, const float* __restrict__ lse2, float* __restrict__ scores) {
+                       Shape sh, Tables tb, const float* __restrict__ nlse, float* __restrict__ scores) {
   extern __shared__ uint8_t smem_raw[];
   P2Smem& sm = *reinterpret_cast<P2Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -312,7 +334,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     for (int i = 0; i < 2; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
     for (int i = 0; i < kQStages; ++i) {
       mbar_init(&sm.q_full[i], 1);
-      mbar_init(&sm.q_empty[i], 1);
+      mbar_init(&sm.q_empty[i], 1 + 4);   // MMA commit + one arrival per consumer warp
       mbar_init(&sm.tm_full[i], 1);
       mbar_init(&sm.tm_empty[i], kTile);
     }
@@ -320,7 +342,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (warp == 2) {
+  if (warp == kProducerWarp) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -330,7 +352,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
-  if (warp == 0 && lane == 0) {
+  if (warp == kProducerWarp && lane == 0) {
     // ---- TMA producer: K tile of layer l, then the C row chunks of layer l
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
@@ -348,16 +370,18 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
       for (int c = 0; c < C; ++c) {
         const int q = l * C + c, qs = q % kQStages;
         if (!mbar_wait(&sm.q_empty[qs], ((q / kQStages) & 1) ^ 1, abort)) { ok = false; break; }
-        mbar_arrive_expect_tx(&sm.q_full[qs], kTileBytes);
+        mbar_arrive_expect_tx(&sm.q_full[qs], kTileBytes + kTile * 4);
         tma_load_2d(sm.q[qs][0], &tmQ, 0, qy0 + c * (int)kTile, &sm.q_full[qs]);
         tma_load_2d(sm.q[qs][1], &tmQ, 64, qy0 + c * (int)kTile, &sm.q_full[qs]);
+        bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C + c) * kTile,
+                  kTile * 4, &sm.q_full[qs]);
         ++q_issued;
       }
     }
     for (int i = max(0, k_issued - 2); i < k_issued; ++i) drain_wait(&sm.k_full[i & 1], (i >> 1) & 1);
     for (int i = max(0, q_issued - kQStages); i < q_issued; ++i)
       drain_wait(&sm.q_full[i % kQStages], (i / kQStages) & 1);
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == kMmaWarp && lane == 0) {
     // ---- MMA issuer: D[key][row] = K_tile . Q_chunk^T
     bool ok = true;
     for (int l = 0; ok && l < L; ++l) {
@@ -369,7 +393,8 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
         if (!mbar_wait(&sm.q_full[qs], use & 1, abort)) { ok = false; break; }
         if (!mbar_wait(&sm.tm_empty[qs], (use & 1) ^ 1, abort)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t idesc = idesc_bf16_f32(kTile, (uint32_t)chunk_cols(rows, c));
+        // always a full 128-row chunk: rows past the row set carry a -inf normaliser
+        const uint32_t idesc = idesc_bf16_f32(kTile, kTile);
         const uint32_t d = tbase + (uint32_t)qs * kTile;
 #pragma unroll
         for (int kb = 0; kb < 2; ++kb)
@@ -384,74 +409,60 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     }
     mma_commit(&sm.mma_done);
     drain_wait(&sm.mma_done, 0);
-  } else if (warp >= 4) {
+  } else if (warp < 8) {
     // ---- column sums: one thread per key (= TMEM lane); warpgroup wg takes
     // the chunks q = l*C + c with q % 2 == wg
-    const int wg = (warp - 4) >> 2;
+    const int wg = warp >> 2;
     const int key = ((warp & 3) << 5) + lane;
     const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
     const float s2 = sh.scale_log2;
     const int v = kt * (int)kTile + key;
     const bool per_layer = sh.rank_mode == VC_RANK_PER_LAYER;
     const int nq = L * C;
-    auto lse_of = [&](int q) -> float {
-      const int l = q / C, c = q % C;
-      const int rho = c * (int)kTile + key;
-      return rho < rows ? lse2[rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho] : INFINITY;
-    };
-    float nxt = wg < nq ? lse_of(wg) : INFINITY;
     Kahan tot, lay;
     tot.init();
     lay.init();
-    int n_mine = 0;
     for (int q = 0; q < nq; ++q) {
       const int l = q / C, c = q % C;
       if ((q & 1) == wg) {
-        // stage this chunk's normalisers for the whole warpgroup
-        float* buf = sm.lse[wg][n_mine & 1];
-        buf[key] = nxt;
-        named_sync(2 + wg, kTile);
-        if (q + 2 < nq) nxt = lse_of(q + 2);
-        ++n_mine;
         const int qs = q % kQStages;
         const uint32_t use = (uint32_t)(q / kQStages);
         const bool go = __all_sync(0xffffffffu, *abort == 0);
         if (go && warp_wait(&sm.tm_full[qs], use & 1, abort)) {
           tc_fence_after();
-          const int ncol = chunk_cols(rows, c);
           const uint32_t col0 = tbase + lane_off + (uint32_t)qs * kTile;
-          for (int p0 = 0; p0 < ncol; p0 += 64) {
-            const int np = min(4, (ncol - p0) >> 4);
-            float x[4][16];
-            {
-              uint32_t v[4][16];
+          float x[8][16];
+          {
+            uint32_t v[8][16];
 #pragma unroll
-              for (int p = 0; p < 4; ++p)
-                if (p < np) tmem_ld16(col0 + p0 + p * 16, v[p]);
-              tmem_wait_only();
+            for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, v[p]);
+            tmem_wait_only();
 #pragma unroll
-              for (int p = 0; p < 4; ++p)
-                if (p < np) {
-                  reg_fence(v[p]);
+            for (int p = 0; p < 8; ++p) {
+              reg_fence(v[p]);
 #pragma unroll
-                  for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
-                }
-            }
-            if (p0 + 64 >= ncol) {
-              tc_fence_before();
-              mbar_arrive(&sm.tm_empty[qs]);
-            }
-#pragma unroll
-            for (int p = 0; p < 4; ++p) {
-              if (p < np) {
-                float e[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) e[j] = ex2(fmaf(x[p][j], s2, -buf[p0 + p * 16 + j]));
-                lay.add(sum16(e));
-              }
+              for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
             }
           }
+          tc_fence_before();
+          mbar_arrive(&sm.tm_empty[qs]);
+          const float4* nl = reinterpret_cast<const float4*>(sm.nlse[qs]);
+          float ps[8];
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {
+            float2 nb[8];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const float4 f = nl[p * 4 + j];
+              nb[2 * j] = make_float2(f.x, f.y);
+              nb[2 * j + 1] = make_float2(f.z, f.w);
+            }
+            ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
+          }
+          lay.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.q_empty[qs]);   // this warp is done with the stage's normalisers
       }
       if (c == C - 1) {
         if (per_layer) {
@@ -475,7 +486,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) {
+  if (warp == kProducerWarp) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tbase, kTmemCols);
@@ -518,7 +529,7 @@ bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows) {
 int score_tc_max_splits() { return 2; }
 
 cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
-                            const TcPlan& tp, float2* part, float* lse2, const float* lse_nat,
+                            const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
                             float* scores, cudaStream_t st) {
   CUtensorMap mq, mk;
   if (!make_rows_map(&mq, Qw, tp.q_rows) || !make_rows_map(&mk, K, tp.k_rows))
@@ -535,8 +546,8 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
   }
   {
     ProfileScope ps("lse_merge", st);
-    lse_merge_kernel<<<dim3((unsigned)((tp.max_rows + 255) / 256), sh.n_req), 256, 0, st>>>(
-        sh, tb, tp.S, part, lse_nat, lse2);
+    lse_merge_kernel<<<dim3((unsigned)((tp.max_prows + 255) / 256), sh.n_req), 256, 0, st>>>(
+        sh, tb, tp.S, part, lse_nat, nlse_pad);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -544,7 +555,7 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
   e = cudaFuncSetAttribute(score_colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   if (e != cudaSuccess) return e;
   ProfileScope ps("score_colsum_tc", st);
-  score_colsum_tc_kernel<<<tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, lse2, scores);
+  score_colsum_tc_kernel<<<tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, nlse_pad, scores);
   return cudaGetLastError();
 }
 

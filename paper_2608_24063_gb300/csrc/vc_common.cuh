@@ -20,6 +20,7 @@ struct Req {                 // one request of a batch
   int64_t s_off;             // float offset of its scores [Hkv][n] or [L][Hkv][n]
   int64_t out_row0;          // first output row (K_out/V_out/idx_out)
   int64_t drop_row0;         // first drop-list row
+  int64_t lsep_off;          // float offset of its chunk-padded row normalisers [L][Hkv][C*128]
   int32_t n, W, Nq, h;
   int32_t C;                 // 128-row chunks of one (layer, KV head) row set, ceil(G*W/128)
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)

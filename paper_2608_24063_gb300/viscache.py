@@ -170,7 +170,7 @@ def prunekv_score(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,
     return scores
 
 
-STATIC_SCRATCH_BYTES = 4 << 20
+STATIC_SCRATCH_BYTES = 16 << 20
 
 
 def prunekv_score_static(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,

@@ -273,12 +273,16 @@ cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, 
                            scores, st);
 }
 
-// Eq. (redistribution, weight_fusion) on tensor cores (bf16, d = 128) or CUDA cores.
-cudaError_t launch_fuse(int dtype, const void* V, const Layout& lay, const Shape& sh,
-                        const Tables& tb, const int32_t* keep, const int32_t* drop, float mu,
-                        float tau, void* V_out, cudaStream_t st) {
+// Prune keys and fuse values, Eq. (redistribution, weight_fusion): one tensor-core
+// kernel for bf16, d = 128 (it also copies the kept keys), else the key gather and
+// the CUDA-core fusion.
+cudaError_t launch_fuse(int dtype, const void* K, const void* V, const Layout& lay,
+                        const Shape& sh, const Tables& tb, const int32_t* keep, const int32_t* drop,
+                        float mu, float tau, void* K_out, void* V_out, cudaStream_t st) {
   if (g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128)
-    return launch_fuse_tc(V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse_tc, st);
+    return launch_fuse_tc(K, V, sh, tb, keep, drop, mu, tau, K_out, V_out, lay.units_fuse_tc, st);
+  cudaError_t e = launch_gather_k(dtype, K, sh, tb, keep, K_out, lay.out_rows, st);
+  if (e != cudaSuccess) return e;
   return launch_fuse_simt(dtype, V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse, st);
 }
 
@@ -455,9 +459,7 @@ int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int
   if (e != cudaSuccess) return VC_ERR_CUDA;
   const Shape sh = lay.shape(1.f);
   const Tables tb = lay.tables(w);
-  e = launch_gather_k(dtype, K, sh, tb, keep_idx, K_out, lay.out_rows, st);
-  if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_fuse(dtype, V, lay, sh, tb, keep_idx, drop_idx, mu, tau, V_out, st);
+  e = launch_fuse(dtype, K, V, lay, sh, tb, keep_idx, drop_idx, mu, tau, K_out, V_out, st);
   return cuda_status(e);
 }
 
@@ -493,9 +495,7 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   e = launch_select(sh, tb, problems, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
                     reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_gather_k(p->dtype, K, sh, tb, idx_out, K_out, lay.out_rows, st);
-  if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_fuse(p->dtype, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, V_out, st);
+  e = launch_fuse(p->dtype, K, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, K_out, V_out, st);
   return cuda_status(e);
 }
 

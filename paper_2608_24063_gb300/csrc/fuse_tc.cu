@@ -1,21 +1,23 @@
-// Value fusion on the tcgen05 tensor cores, Eq. (redistribution) and
-// Eq. (weight_fusion); bf16 inputs, d = 128.
+// Key pruning and value fusion on the tcgen05 tensor cores, Eq. (redistribution)
+// and Eq. (weight_fusion); bf16 inputs, d = 128.
 //
-// One CTA per (request, layer, KV head, tile of 128 kept rows):
-//   O = softmax_row(V_k V_d^T / tau) V_d, online over tiles of 128 dropped rows,
-//   V_out = mu V_k + (1 - mu) O.
-// Kept and dropped rows are gathered by index with cp.async into 128-byte
-// swizzled tiles (the layout TMA would write).  S = V_k V_d^T and
-// O += P V_d run on tcgen05.mma with fp32 accumulators in tensor memory:
-// V_d is read K-major for the first product and MN-major for the second;
-// P goes through shared memory in bf16.  The softmax keeps a per-row
-// reference maximum and only rescales O (in tensor memory) when a tile's
-// maximum exceeds it by more than 2^8, so rescaling is rare.
+// One CTA per (request, layer, KV head, tile of 256 kept rows):
+//   K_out = K[keep]                                   (bit-exact row copy)
+//   O     = softmax_row(V_k V_d^T / tau) V_d          (online over tiles of 128 dropped rows)
+//   V_out = mu V_k + (1 - mu) O
+// Kept and dropped value rows are gathered by index with cp.async into
+// 128-byte swizzled tiles (the layout TMA would write).  S = V_k V_d^T and
+// O += P V_d run on tcgen05.mma with fp32 accumulators in tensor memory; V_d
+// is read K-major for the first product and MN-major for the second, P goes
+// through shared memory in bf16.  The two halves of the kept tile (two
+// consumer warpgroups) share every gathered V_d tile.  The softmax keeps a
+// per-row reference maximum and rescales O (in tensor memory) only when a
+// tile's maximum exceeds it by more than 2^8.
 //
-// Warp roles (256 threads, one CTA per SM): warp 0 allocates tensor memory
-// and one of its threads issues the MMAs; warps 1-3 gather rows; warps 4-7
-// own one kept row each (= TMEM lane) for the softmax and the epilogue.
-// Every wait is bounded (see tc_common.cuh).
+// Warp roles (384 threads, one CTA per SM): warps 0-3 and 4-7 own one kept
+// row each (= TMEM lane) for the softmax and the epilogue, warps 8-10 gather
+// rows and copy the kept keys, warp 11 allocates tensor memory and one of its
+// threads issues the MMAs.  Every wait is bounded (see tc_common.cuh).
 #include "kernels.h"
 #include "profile.h"
 #include "tc_common.cuh"
@@ -26,19 +28,21 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 256;
-constexpr int kProducers = 96;                   // warps 1-3
+constexpr int kThreads = 384;
+constexpr int kProducers = 96;                   // warps 8-10
+constexpr int kMmaWarp = 11;
 constexpr uint32_t kTile = 128;
 constexpr uint32_t kKB = kTile * 128;            // one K-block: 128 rows x 128 bytes
 constexpr int kVdStages = 3;
-constexpr uint32_t kTmemCols = 512;              // O: 0..127, S: 128..383
+constexpr int kKChunks = (2 * 128 * 16 + kProducers - 1) / kProducers;   // kept-row chunks per producer
+constexpr uint32_t kTmemCols = 512;              // O_0, O_1, S_0, S_1: 128 columns each
 constexpr float kRescaleLog2 = 8.f;
 
 struct FSmem {
-  uint8_t vk[2][kKB];                 // kept rows: A operand of S = V_k V_d^T
+  uint8_t vk[2][2][kKB];              // [half][K-block] kept rows: A operand of S = V_k V_d^T
   uint8_t vd[kVdStages][2][kKB];      // dropped rows: B operand of both products
-  uint8_t p[2][2][kKB];               // softmax numerators (bf16): A operand of O += P V_d
-  int32_t idx[1 + kVdStages][kTile];  // row positions of the kept tile and of each drop stage
+  uint8_t p[2][2][kKB];               // [half][K-block] numerators (bf16): A of O += P V_d
+  int32_t idx_d[kVdStages][kTile];    // dropped positions of each stage
   uint64_t vk_full;
   uint64_t vd_full[kVdStages], vd_empty[kVdStages];
   uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
@@ -68,9 +72,9 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
   return (uint32_t)((c >> 3) * kKB + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
 
-// Row position r of a tile whose positions are pos[0..count): -1 (zero row)
-// beyond count or for a position outside [0, n) (recorded in the status word).
-__device__ __forceinline__ int32_t tile_pos(const int32_t* pos, int count, int r, int n,
+// Position r of a list pos[0..count): -1 beyond count or outside [0, n)
+// (the latter recorded in the status word).
+__device__ __forceinline__ int32_t list_pos(const int32_t* pos, int count, int r, int n,
                                             int32_t* status) {
   if (r >= count) return -1;
   const int32_t v = pos[r];
@@ -92,15 +96,45 @@ __device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* s
   }
 }
 
+// K_out rows of the tile: bit-exact 16-byte copies of the kept key rows.
+// Producer thread tid owns chunks e = tid + kProducers * i of the 256-row tile,
+// whose row positions it holds in kpos[i] (-1 = no row).
+__device__ __forceinline__ void copy_keys(__nv_bfloat16* K_out, int64_t orow,
+                                          const __nv_bfloat16* Kl, const int32_t (&kpos)[kKChunks],
+                                          int tid) {
+#pragma unroll
+  for (int i = 0; i < kKChunks; ++i) {
+    const int e = tid + kProducers * i;
+    if (kpos[i] >= 0)
+      reinterpret_cast<uint4*>(K_out + (orow + (e >> 4)) * 128)[e & 15] =
+          reinterpret_cast<const uint4*>(Kl + (int64_t)kpos[i] * 128)[e & 15];
+  }
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// 64 consecutive TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_cols64(uint32_t taddr, float (&x)[4][16]) {
+  uint32_t v[4][16];
+#pragma unroll
+  for (int p = 0; p < 4; ++p) tmem_ld16(taddr + p * 16, v[p]);
+  tmem_wait_only();
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    reg_fence(v[p]);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
-                 const int32_t* __restrict__ keep_idx, const int32_t* __restrict__ drop_idx,
-                 float mu, float c2, __nv_bfloat16* __restrict__ V_out) {
+fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
+                 Shape sh, Tables tb, const int32_t* __restrict__ keep_idx,
+                 const int32_t* __restrict__ drop_idx, float mu, float c2,
+                 __nv_bfloat16* __restrict__ K_out, __nv_bfloat16* __restrict__ V_out) {
   extern __shared__ uint8_t smem_raw[];
   FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -109,15 +143,18 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
   const int r = rl / sh.L, l = rl % sh.L;
   const Req rq = tb.req[r];
   const Layer ly = tb.layer[rl];
-  const int ktiles = (ly.B + (int)kTile - 1) / (int)kTile;
+  const int ktiles = (ly.B + 2 * (int)kTile - 1) / (2 * (int)kTile);
   const int u = blockIdx.x - tb.unit0_fuse_tc[rl];
   const int g = u / ktiles;
-  const int r0 = (u % ktiles) * (int)kTile;
-  const int rows = min((int)kTile, ly.B - r0);
+  const int r0 = (u % ktiles) * 2 * (int)kTile;
+  const int rows = min(2 * (int)kTile, ly.B - r0);        // kept rows of this CTA
+  const int nhalf = rows > (int)kTile ? 2 : 1;            // halves with kept rows
   const int D = ly.D;
   const int nt = (D + (int)kTile - 1) / (int)kTile;
 
-  const __nv_bfloat16* Vl = V + rq.kv_off + ((int64_t)l * sh.Hkv + g) * rq.n * 128;
+  const int64_t slab = ((int64_t)l * sh.Hkv + g) * rq.n * 128;
+  const __nv_bfloat16* Vl = V + rq.kv_off + slab;
+  const __nv_bfloat16* Kl = K + rq.kv_off + slab;
   const int64_t orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
   const int32_t* kp = keep_idx + orow;
   const int32_t* dp = drop_idx + rq.drop_row0 + (int64_t)sh.Hkv * ly.Qd + (int64_t)g * D;
@@ -136,7 +173,7 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (warp == 0) {
+  if (warp == kMmaWarp) {
     tmem_alloc(&sm.tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -146,72 +183,95 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
-  if (warp == 0) {
+  if (warp == kMmaWarp) {
     if (lane == 0) {
-      // ---- MMA issuer
+      // ---- MMA issuer.  Per drop tile j: S_h = V_k,h V_d(j)^T for both halves,
+      // then O_h += P_h(j-1) V_d(j-1) for both halves.
       const uint32_t id_s = idesc_bf16_f32(kTile, kTile);
       const uint32_t id_o = idesc_bf16_f32_bmn(kTile, kTile);
       bool ok = mbar_wait(&sm.vk_full, 0, abort);
       for (int j = 0; ok && j <= nt; ++j) {
         if (j < nt) {
-          const int st = j % kVdStages, sb = j & 1;
+          const int st = j % kVdStages;
           if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
-          if (!mbar_wait(&sm.s_empty[sb], ((j >> 1) & 1) ^ 1, abort)) break;
-          tc_fence_after();
-          const uint32_t d = tbase + kTile + (uint32_t)sb * kTile;
+          for (int h = 0; h < nhalf && ok; ++h) {
+            if (!mbar_wait(&sm.s_empty[h], (j & 1) ^ 1, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t d = tbase + (uint32_t)(2 + h) * kTile;
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            mma_bf16(d, desc_sw128(smem_u32(sm.vk[kk >> 2]) + (kk & 3) * 32),
-                     desc_sw128(smem_u32(sm.vd[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
-          mma_commit(&sm.s_full[sb]);
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16(d, desc_sw128(smem_u32(sm.vk[h][kk >> 2]) + (kk & 3) * 32),
+                       desc_sw128(smem_u32(sm.vd[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
+            mma_commit(&sm.s_full[h]);
+          }
+          if (!ok) break;
         }
         if (j >= 1) {
-          const int jp = j - 1, pb = jp & 1, st = jp % kVdStages;
-          if (!mbar_wait(&sm.p_full[pb], (jp >> 1) & 1, abort)) break;
-          tc_fence_after();
+          const int jp = j - 1, st = jp % kVdStages;
+          for (int h = 0; h < nhalf && ok; ++h) {
+            if (!mbar_wait(&sm.p_full[h], jp & 1, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t d = tbase + (uint32_t)h * kTile;
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-            mma_bf16(tbase, desc_sw128(smem_u32(sm.p[pb][kk >> 2]) + (kk & 3) * 32),
-                     desc_sw128_mn(smem_u32(sm.vd[st][0]) + kk * 2048, kKB), id_o,
-                     (jp > 0 || kk > 0) ? 1u : 0u);
-          mma_commit(&sm.p_empty[pb]);
-          mma_commit(&sm.vd_empty[st]);
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16(d, desc_sw128(smem_u32(sm.p[h][kk >> 2]) + (kk & 3) * 32),
+                       desc_sw128_mn(smem_u32(sm.vd[st][0]) + kk * 2048, kKB), id_o,
+                       (jp > 0 || kk > 0) ? 1u : 0u);
+            mma_commit(&sm.p_empty[h]);
+          }
+          if (ok) mma_commit(&sm.vd_empty[st]);
         }
       }
       mma_commit(&sm.o_full);
       mma_commit(&sm.mma_done);
       drain_wait(&sm.mma_done, 0);
     }
-  } else if (warp < 4) {
-    // ---- row gathers (cp.async).  The positions of a tile go to shared memory
-    // first (fetched one tile ahead), so the copies issue back to back; a
-    // stage is published once its copies landed.
-    const int tid = threadIdx.x - 32;
-    sm.idx[0][tid] = tile_pos(kp, rows, tid, rq.n, tb.status);
-    if (tid + kProducers < (int)kTile) sm.idx[0][tid + kProducers] = tile_pos(kp, rows, tid + kProducers, rq.n, tb.status);
-    named_sync(1, kProducers);
-    gather_tile(&sm.vk[0][0], Vl, sm.idx[0], tid);
+  } else if (warp >= 8) {
+    // ---- row gathers (cp.async) and the key copy.  Positions go to shared
+    // memory first (the next tile's fetched one tile ahead) so the copies issue
+    // back to back; a stage is published once its copies landed.
+    const int tid = threadIdx.x - 256;
+    int32_t kpos[kKChunks];                      // positions of this thread's kept-row chunks
+#pragma unroll
+    for (int i = 0; i < kKChunks; ++i) {
+      const int e = tid + kProducers * i;
+      kpos[i] = e < 2 * (int)kTile * 16 ? list_pos(kp, rows, e >> 4, rq.n, tb.status) : -1;
+    }
+#pragma unroll
+    for (int i = 0; i < kKChunks; ++i) {
+      const int e = tid + kProducers * i;
+      if (e < 2 * (int)kTile * 16) {
+        const int rr = e >> 4, c = e & 15;
+        cp_async16(&sm.vk[rr >> 7][0][0] + swz(rr & 127, c), kpos[i] >= 0 ? Vl + (int64_t)kpos[i] * 128 + c * 8 : Vl,
+                   kpos[i] >= 0 ? 16u : 0u);
+      }
+    }
     cp_async_commit();
     cp_async_wait<0>();
     fence_proxy_async();
     mbar_arrive(&sm.vk_full);
-    int cnt = min((int)kTile, D);
-    int32_t a0 = nt > 0 ? tile_pos(dp, cnt, tid, rq.n, tb.status) : -1;
-    int32_t a1 = nt > 0 && tid + kProducers < (int)kTile ? tile_pos(dp, cnt, tid + kProducers, rq.n, tb.status) : -1;
+    int32_t a0 = -1, a1 = -1;
+    if (nt > 0) {
+      const int cnt = min((int)kTile, D);
+      a0 = list_pos(dp, cnt, tid, rq.n, tb.status);
+      a1 = tid + kProducers < (int)kTile ? list_pos(dp, cnt, tid + kProducers, rq.n, tb.status) : -1;
+    }
+    bool keys_done = false;
     int j = 0;
     for (; j < nt; ++j) {
       const int st = j % kVdStages;
-      int32_t* buf = sm.idx[1 + st];
+      int32_t* buf = sm.idx_d[st];
+      if (tid == 0) sm.gather_go = mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort) ? 1 : 0;
+      named_sync(1, kProducers);                 // the stage is free and its old positions unread
+      if (!sm.gather_go) break;
       buf[tid] = a0;
       if (tid + kProducers < (int)kTile) buf[tid + kProducers] = a1;
-      if (tid == 0) sm.gather_go = mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort) ? 1 : 0;
       named_sync(1, kProducers);
-      if (!sm.gather_go) break;
       if (j + 1 < nt) {
         const int32_t* nxt = dp + (j + 1) * (int)kTile;
-        cnt = min((int)kTile, D - (j + 1) * (int)kTile);
-        a0 = tile_pos(nxt, cnt, tid, rq.n, tb.status);
-        a1 = tid + kProducers < (int)kTile ? tile_pos(nxt, cnt, tid + kProducers, rq.n, tb.status) : -1;
+        const int cnt = min((int)kTile, D - (j + 1) * (int)kTile);
+        a0 = list_pos(nxt, cnt, tid, rq.n, tb.status);
+        a1 = tid + kProducers < (int)kTile ? list_pos(nxt, cnt, tid + kProducers, rq.n, tb.status) : -1;
       }
       gather_tile(&sm.vd[st][0][0], Vl, buf, tid);
       cp_async_commit();
@@ -219,45 +279,47 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
         cp_async_wait<1>();
         fence_proxy_async();
         mbar_arrive(&sm.vd_full[(j - 1) % kVdStages]);
+        if (!keys_done) {                        // while the first products run
+          copy_keys(K_out, orow, Kl, kpos, tid);
+          keys_done = true;
+        }
       }
     }
     cp_async_wait<0>();
     fence_proxy_async();
     if (j >= 1) mbar_arrive(&sm.vd_full[(j - 1) % kVdStages]);
+    if (!keys_done) copy_keys(K_out, orow, Kl, kpos, tid);
   } else {
     // ---- softmax over the drop set and epilogue: one thread per kept row
-    const int row = threadIdx.x - 128;
+    const int h = warp >> 2;                              // half of the kept tile
+    const int row = ((warp & 3) << 5) + lane;             // row within the half = TMEM lane
     const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    const uint32_t o_col = tbase + lane_off + (uint32_t)h * kTile;
+    const uint32_t s_col = tbase + lane_off + (uint32_t)(2 + h) * kTile;
+    const bool active = h < nhalf;
     float m = -INFINITY, lsum = 0.f;
     bool ok = true;
-    for (int j = 0; j < nt; ++j) {
-      const int sb = j & 1;
-      if (!warp_wait(&sm.s_full[sb], (j >> 1) & 1, abort)) { ok = false; break; }
+    for (int j = 0; active && j < nt; ++j) {
+      if (!warp_wait(&sm.s_full[h], j & 1, abort)) { ok = false; break; }
       tc_fence_after();
-      float x[8][16];
-      {
-        uint32_t v[8][16];
-#pragma unroll
-        for (int p = 0; p < 8; ++p) tmem_ld16(tbase + lane_off + kTile + sb * kTile + p * 16, v[p]);
-        tmem_wait_only();
-#pragma unroll
-        for (int p = 0; p < 8; ++p) {
-          reg_fence(v[p]);
-#pragma unroll
-          for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
-        }
-      }
-      tc_fence_before();
-      mbar_arrive(&sm.s_empty[sb]);
       const int valid = min((int)kTile, D - j * (int)kTile);
+      // pass A over S: the tile maximum
       float tm = -INFINITY;
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {
+        float x[4][16];
+        tmem_cols64(s_col + hh * 64, x);
+        float pm[4];
 #pragma unroll
-      for (int p = 0; p < 8; ++p)
+        for (int p = 0; p < 4; ++p) {
+          float a = -INFINITY;
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          if (p * 16 + q >= valid) x[p][q] = -INFINITY;
-          tm = fmaxf(tm, x[p][q]);
+          for (int q = 0; q < 16; ++q)
+            if (hh * 64 + p * 16 + q < valid) a = fmaxf(a, x[p][q]);
+          pm[p] = a;
         }
+        tm = fmax3(tm, fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3]));
+      }
       tm *= c2;
       // raise the reference maximum when this tile exceeds it by more than 2^8
       const bool raise = tm > m + kRescaleLog2;
@@ -265,96 +327,109 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
       const float corr = raise ? ex2(m - m_new) : 1.f;     // 0 on the first tile
       if (__any_sync(0xffffffffu, raise && j > 0)) {
         // O holds the tiles before j: wait for their last product, then rescale in place
-        if (!warp_wait(&sm.p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) { ok = false; break; }
+        if (!warp_wait(&sm.p_empty[h], (j - 1) & 1, abort)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
+        for (int hh = 0; hh < 2; ++hh) {
           uint32_t v[4][16];
 #pragma unroll
-          for (int p = 0; p < 4; ++p) tmem_ld16(tbase + lane_off + (h * 4 + p) * 16, v[p]);
+          for (int p = 0; p < 4; ++p) tmem_ld16(o_col + hh * 64 + p * 16, v[p]);
           tmem_wait_only();
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
             reg_fence(v[p]);
 #pragma unroll
             for (int q = 0; q < 16; ++q) v[p][q] = __float_as_uint(__uint_as_float(v[p][q]) * corr);
-            tmem_st16(tbase + lane_off + (h * 4 + p) * 16, v[p]);
+            tmem_st16(o_col + hh * 64 + p * 16, v[p]);
           }
         }
         tmem_wait_st();
       }
       lsum *= corr;
       m = m_new;
-      // numerators in bf16 into the P tile (row-major, swizzled, K-major A operand)
-      if (!warp_wait(&sm.p_empty[sb], ((j >> 1) & 1) ^ 1, abort)) { ok = false; break; }
-      uint8_t* pt = &sm.p[sb][0][0];
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        float e[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          e[q] = ex2(fmaf(x[c >> 1][(c & 1) * 8 + q], c2, -m));
-          lsum += e[q];
+      // the P tile is free once the previous product has read it
+      if (!warp_wait(&sm.p_empty[h], (j & 1) ^ 1, abort)) { ok = false; break; }
+      // pass B over S: numerators in bf16 into the P tile (swizzled K-major A operand)
+      uint8_t* pt = &sm.p[h][0][0];
+      float2 ls = make_float2(0.f, 0.f);
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {
+        float x[4][16];
+        tmem_cols64(s_col + hh * 64, x);
+        if (hh == 1) {
+          tc_fence_before();
+          mbar_arrive(&sm.s_empty[h]);             // S copied out: the next product may start
         }
-        uint4 w;
-        w.x = pack_bf16x2(e[0], e[1]);
-        w.y = pack_bf16x2(e[2], e[3]);
-        w.z = pack_bf16x2(e[4], e[5]);
-        w.w = pack_bf16x2(e[6], e[7]);
-        *reinterpret_cast<uint4*>(pt + swz(row, c)) = w;
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+#pragma unroll
+          for (int c8 = 0; c8 < 2; ++c8) {
+            float e[8];
+#pragma unroll
+            for (int q = 0; q < 8; q += 2) {
+              const int col = hh * 64 + p * 16 + c8 * 8 + q;
+              const float2 t = __ffma2_rn(make_float2(x[p][c8 * 8 + q], x[p][c8 * 8 + q + 1]),
+                                          make_float2(c2, c2), make_float2(-m, -m));
+              e[q] = col < valid ? ex2(t.x) : 0.f;
+              e[q + 1] = col + 1 < valid ? ex2(t.y) : 0.f;
+              ls = __fadd2_rn(ls, make_float2(e[q], e[q + 1]));
+            }
+            uint4 w;
+            w.x = pack_bf16x2(e[0], e[1]);
+            w.y = pack_bf16x2(e[2], e[3]);
+            w.z = pack_bf16x2(e[4], e[5]);
+            w.w = pack_bf16x2(e[6], e[7]);
+            *reinterpret_cast<uint4*>(pt + swz(row, hh * 8 + p * 2 + c8)) = w;
+          }
+        }
       }
+      lsum += ls.x + ls.y;
       fence_proxy_async();
       tc_fence_before();
-      mbar_arrive(&sm.p_full[sb]);
+      mbar_arrive(&sm.p_full[h]);
     }
     // epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped;
     // the kept rows are read from shared memory once their gather has landed
     const bool have_k = warp_wait(&sm.vk_full, 0, abort);
-    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
+    const bool have_o = active && have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
     if (have_o) tc_fence_after();
     const float w_o = have_o ? (1.f - mu) / lsum : 0.f;
     const float w_k = have_o ? mu : 1.f;
-    uint32_t ov[8][16];
-    if (have_o) {
+    const int grow = h * (int)kTile + row;                // row within the CTA's kept tile
+#pragma unroll 1
+    for (int hh = 0; hh < 2; ++hh) {
+      float o[4][16];
+      if (have_o) {
+        tmem_cols64(o_col + hh * 64, o);
+      } else {
 #pragma unroll
-      for (int p = 0; p < 8; ++p) tmem_ld16(tbase + lane_off + p * 16, ov[p]);
-      tmem_wait_only();
+        for (int p = 0; p < 4; ++p)
 #pragma unroll
-      for (int p = 0; p < 8; ++p) reg_fence(ov[p]);
-    } else {
+          for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
+      }
+      if (have_k && grow < rows) {
 #pragma unroll
-      for (int p = 0; p < 8; ++p)
-#pragma unroll
-        for (int q = 0; q < 16; ++q) ov[p][q] = 0u;
-    }
-#pragma unroll
-    for (int p = 0; p < 8; ++p) {
-      float o[16];
-#pragma unroll
-      for (int q = 0; q < 16; ++q) o[q] = __uint_as_float(ov[p][q]);
-      if (have_k && row < rows) {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int c = p * 2 + h;
-          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[0][0] + swz(row, c));
+        for (int c8 = 0; c8 < 8; ++c8) {
+          const int c = hh * 8 + c8;
+          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[h][0][0] + swz(row, c));
           const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
           uint4 w;
           uint32_t* wp = &w.x;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float2 kf = __bfloat1622float2(k2[q]);
-            const float a = fmaf(w_k, kf.x, w_o * o[h * 8 + 2 * q]);
-            const float b = fmaf(w_k, kf.y, w_o * o[h * 8 + 2 * q + 1]);
+            const float a = fmaf(w_k, kf.x, w_o * o[c8 >> 1][(c8 & 1) * 8 + 2 * q]);
+            const float b = fmaf(w_k, kf.y, w_o * o[c8 >> 1][(c8 & 1) * 8 + 2 * q + 1]);
             wp[q] = pack_bf16x2(a, b);
           }
-          *reinterpret_cast<uint4*>(V_out + (orow + row) * 128 + c * 8) = w;
+          *reinterpret_cast<uint4*>(V_out + (orow + grow) * 128 + c * 8) = w;
         }
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == kMmaWarp) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tbase, kTmemCols);
@@ -364,19 +439,20 @@ fuse_v_tc_kernel(const __nv_bfloat16* __restrict__ V, Shape sh, Tables tb,
 
 }  // namespace
 
-int fuse_rows_per_tile_tc() { return (int)kTile; }
+int fuse_rows_per_tile_tc() { return 2 * (int)kTile; }
 
-cudaError_t launch_fuse_tc(const void* V, const Shape& sh, const Tables& tb,
+cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const Tables& tb,
                            const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
-                           void* V_out, int units, cudaStream_t st) {
+                           void* K_out, void* V_out, int units, cudaStream_t st) {
   if (units == 0) return cudaSuccess;
   const size_t smem = sizeof(FSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(fuse_v_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  ProfileScope ps("fuse_v_tc", st);
+  ProfileScope ps("fuse_kv_tc", st);
   fuse_v_tc_kernel<<<units, kThreads, smem, st>>>(
-      static_cast<const __nv_bfloat16*>(V), sh, tb, keep_idx, drop_idx, mu, kLog2e / tau,
+      static_cast<const __nv_bfloat16*>(K), static_cast<const __nv_bfloat16*>(V), sh, tb, keep_idx,
+      drop_idx, mu, kLog2e / tau, static_cast<__nv_bfloat16*>(K_out),
       static_cast<__nv_bfloat16*>(V_out));
   return cudaGetLastError();
 }

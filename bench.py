@@ -96,7 +96,8 @@ KERNEL_WORK = {
     "score_lse_tc": ("tensor", "flops_score"),
     "score_colsum_tc": ("tensor", "flops_score"),
     "fuse_v_simt": ("tensor", "flops_fuse"),
-    "fuse_kv_tc": ("tensor", "flops_fuse"),
+    "fuse_v_tc": ("tensor", "flops_fuse"),
+    "gather_kv": ("hbm", "gather_bytes"),
     "gather_k": ("hbm", "gather_bytes"),
 }
 

@@ -174,9 +174,11 @@ int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis,
  *   keep_idx/drop_idx device lists from prunekv_select
  *   mu in [0, 1], tau > 0
  *   K_out, V_out      device, dense varlen (rows Hkv * sum_l B_l, d columns)
- *   ws                workspace of prunekv_fuse_workspace_size(L) bytes
+ *   ws                workspace of prunekv_fuse_workspace_size(B, L, Hkv, d, n, Nq) bytes
+ *                     (bf16, d = 128 also compacts the survivors' values there)
  */
-size_t prunekv_fuse_workspace_size(int32_t L);
+size_t prunekv_fuse_workspace_size(const int32_t* B, int32_t L, int32_t Hkv, int32_t d,
+                                   int32_t n_vis, int32_t Nq);
 int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int32_t Hkv,
                          int32_t d, int32_t n_vis, const int32_t* B, int32_t Nq,
                          const int32_t* keep_idx, const int32_t* drop_idx, float mu,

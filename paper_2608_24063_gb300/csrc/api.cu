@@ -49,18 +49,19 @@ struct RequestPlan {
 struct Layout {
   // inputs
   int n_req = 0, L = 0, Hq = 0, Hkv = 0, d = 0, rank_mode = VC_RANK_SHARED;
-  bool need_lse = false, need_scores = false, need_sort = false, need_drop = false;
+  bool need_lse = false, need_scores = false, need_sort = false, need_drop = false, need_vs = false;
   // tensor-core score plan
   int S = 1;
   int64_t q_rows = 0, k_rows = 0, max_rows = 0, prows = 0, max_prows = 0;
-  std::vector<int32_t> u_tc1, u_tc2, base_tc1, u_fuse_tc;
-  int units_fuse_tc = 0;
+  std::vector<int32_t> u_tc1, u_tc2, base_tc1, u_fuse_tc, u_gather;
+  int units_fuse_tc = 0, units_gather = 0;
+  int64_t vs_rows = 0;
   // derived sizes
   int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
   int units_lse = 0, units_col = 0, units_fuse = 0;
   // workspace offsets
   size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
-         o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, o_u_fuse_tc = 0, table_begin = 0, table_end = 0, o_lse = 0,
+         o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, o_u_fuse_tc = 0, o_u_gather = 0, o_vs = 0, table_begin = 0, table_end = 0, o_lse = 0,
          o_part = 0, o_lsep = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
   // host images
   std::vector<Req> req;
@@ -79,6 +80,8 @@ struct Layout {
     row0.assign((size_t)n_req * L + 1, 0);
     u_tc1.assign(n_req + 1, 0);
     u_fuse_tc.assign((size_t)n_req * L + 1, 0);
+    u_gather.assign((size_t)n_req * L + 1, 0);
+    vs_rows = 0;
     u_tc2.assign(n_req + 1, 0);
     base_tc1.assign(n_req, 0);
     q_rows = k_rows = max_rows = prows = max_prows = 0;
@@ -87,6 +90,7 @@ struct Layout {
     const int rows_tile = score_rows_per_tile_simt(), keys_tile = score_keys_per_tile_simt();
     const int fuse_tile = fuse_rows_per_tile_simt();
     const int fuse_tile_tc = fuse_rows_per_tile_tc();
+    const int gather_rows = gather_rows_per_block();
     for (int r = 0; r < n_req; ++r) {
       const RequestPlan& p = plans[r];
       Req& q = req[r];
@@ -99,6 +103,7 @@ struct Layout {
       q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
       q.C = (G * p.W + 127) / 128;
       q.lsep_off = prows;
+      q.vs_row0 = vs_rows;
       prows += (int64_t)L * Hkv * q.C * 128;
       max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
       q.nrb = (G * p.W + 255) / 256;
@@ -119,6 +124,8 @@ struct Layout {
         row0[rl] = out_rows + (int64_t)Hkv * P;
         u_fuse[rl + 1] = u_fuse[rl] + Hkv * ((b + fuse_tile - 1) / fuse_tile);
         u_fuse_tc[rl + 1] = u_fuse_tc[rl] + Hkv * ((b + fuse_tile_tc - 1) / fuse_tile_tc);
+        u_gather[rl + 1] = u_gather[rl] + Hkv * ((b + ly.D + gather_rows - 1) / gather_rows);
+        vs_rows += (int64_t)Hkv * (b + ly.D);
         P += b;
         Qd += ly.D;
       }
@@ -134,6 +141,7 @@ struct Layout {
     units_col = u_col[n_req];
     units_fuse = u_fuse[(size_t)n_req * L];
     units_fuse_tc = u_fuse_tc[(size_t)n_req * L];
+    units_gather = u_gather[(size_t)n_req * L];
     set_splits(1);
 
     Arena a;
@@ -148,6 +156,7 @@ struct Layout {
     o_u_tc1 = a.take(sizeof(int32_t) * u_tc1.size());
     o_u_tc2 = a.take(sizeof(int32_t) * u_tc2.size());
     o_u_fuse_tc = a.take(sizeof(int32_t) * u_fuse_tc.size());
+    o_u_gather = a.take(sizeof(int32_t) * u_gather.size());
     table_end = a.off;
     if (need_lse) {
       // CUDA-core path: lse rows; tensor-core path: split partials (same region)
@@ -162,6 +171,7 @@ struct Layout {
       if (need_scores) o_rank = a.take(sizeof(int32_t) * score_elems);
     }
     if (need_drop) o_drop = a.take(sizeof(int32_t) * drop_rows);
+    if (need_vs) o_vs = a.take((size_t)256 * std::max<int64_t>(vs_rows, 1));
     total = a.off;
   }
 
@@ -229,6 +239,7 @@ struct Layout {
     put(o_u_tc1, u_tc1.data(), sizeof(int32_t) * u_tc1.size());
     put(o_u_tc2, u_tc2.data(), sizeof(int32_t) * u_tc2.size());
     put(o_u_fuse_tc, u_fuse_tc.data(), sizeof(int32_t) * u_fuse_tc.size());
+    put(o_u_gather, u_gather.data(), sizeof(int32_t) * u_gather.size());
   }
 
   Tables tables(uint8_t* ws) const {
@@ -242,6 +253,7 @@ struct Layout {
     t.unit0_tc1 = reinterpret_cast<const int32_t*>(ws + o_u_tc1);
     t.unit0_tc2 = reinterpret_cast<const int32_t*>(ws + o_u_tc2);
     t.unit0_fuse_tc = reinterpret_cast<const int32_t*>(ws + o_u_fuse_tc);
+    t.unit0_gather = reinterpret_cast<const int32_t*>(ws + o_u_gather);
     t.status = reinterpret_cast<int32_t*>(ws + o_status);
     return t;
   }
@@ -278,9 +290,10 @@ cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, 
 // the CUDA-core fusion.
 cudaError_t launch_fuse(int dtype, const void* K, const void* V, const Layout& lay,
                         const Shape& sh, const Tables& tb, const int32_t* keep, const int32_t* drop,
-                        float mu, float tau, void* K_out, void* V_out, cudaStream_t st) {
-  if (g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128)
-    return launch_fuse_tc(K, V, sh, tb, keep, drop, mu, tau, K_out, V_out, lay.units_fuse_tc, st);
+                        float mu, float tau, void* K_out, void* V_out, uint8_t* w, cudaStream_t st) {
+  if (g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128 && lay.need_vs)
+    return launch_fuse_tc(K, V, sh, tb, keep, drop, mu, tau, K_out, V_out, w + lay.o_vs,
+                          lay.vs_rows, lay.units_gather, lay.units_fuse_tc, st);
   cudaError_t e = launch_gather_k(dtype, K, sh, tb, keep, K_out, lay.out_rows, st);
   if (e != cudaSuccess) return e;
   return launch_fuse_simt(dtype, V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse, st);
@@ -333,6 +346,7 @@ Layout select_layout(int L, int Hkv, int n, const int32_t* B, int Nq, int rank_m
 Layout fuse_layout(int L, int Hkv, int d, int n, const int32_t* B, int Nq) {
   Layout lay;
   lay.L = L; lay.Hq = Hkv; lay.Hkv = Hkv; lay.d = d;
+  lay.need_vs = d == 128;
   RequestPlan p;
   p.n = n; p.W = 1; p.Nq = Nq;
   if (B) p.B.assign(B, B + L);
@@ -365,6 +379,7 @@ Layout compress_layout(const vc_params* p, const std::vector<RequestPlan>& plans
   Layout lay;
   lay.L = p->L; lay.Hq = p->Hq; lay.Hkv = p->Hkv; lay.d = p->d; lay.rank_mode = p->rank_mode;
   lay.need_lse = lay.need_scores = lay.need_sort = lay.need_drop = true;
+  lay.need_vs = p->dtype == VC_BF16 && p->d == 128;
   lay.build(plans);
   return lay;
 }
@@ -435,9 +450,10 @@ int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis, c
   return cuda_status(e);
 }
 
-size_t prunekv_fuse_workspace_size(int32_t L) {
-  if (L < 1 || L > 256) return 0;
-  return fuse_layout(L, 1, 64, 1, nullptr, 0).total;
+size_t prunekv_fuse_workspace_size(const int32_t* B, int32_t L, int32_t Hkv, int32_t d,
+                                   int32_t n_vis, int32_t Nq) {
+  if (L < 1 || L > 256 || Hkv < 1 || (d != 64 && d != 128) || !valid_budgets(B, L, Nq, n_vis)) return 0;
+  return fuse_layout(L, Hkv, d, n_vis, B, Nq).total;
 }
 
 int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int32_t Hkv,
@@ -459,7 +475,7 @@ int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int
   if (e != cudaSuccess) return VC_ERR_CUDA;
   const Shape sh = lay.shape(1.f);
   const Tables tb = lay.tables(w);
-  e = launch_fuse(dtype, K, V, lay, sh, tb, keep_idx, drop_idx, mu, tau, K_out, V_out, st);
+  e = launch_fuse(dtype, K, V, lay, sh, tb, keep_idx, drop_idx, mu, tau, K_out, V_out, w, st);
   return cuda_status(e);
 }
 
@@ -495,7 +511,7 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   e = launch_select(sh, tb, problems, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
                     reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
-  e = launch_fuse(p->dtype, K, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, K_out, V_out, st);
+  e = launch_fuse(p->dtype, K, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, K_out, V_out, w, st);
   return cuda_status(e);
 }
 

@@ -39,12 +39,14 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
                             const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
                             float* scores, cudaStream_t st);
 
-// V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on tcgen05 tensor cores (bf16, d = 128).
+// bf16, d = 128: K_out = K[keep] and the survivors' values compacted into Vs
+// (gather), then V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on tcgen05.
 int fuse_rows_per_tile_tc();
-// (also writes K_out = K[keep])
+int gather_rows_per_block();
 cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const Tables& tb,
                            const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
-                           void* K_out, void* V_out, int units, cudaStream_t st);
+                           void* K_out, void* V_out, void* Vs, int64_t vs_rows, int units_gather,
+                           int units, cudaStream_t st);
 
 // Ranking (radix sort per problem) and ascending keep/drop compaction.
 cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, const float* scores,

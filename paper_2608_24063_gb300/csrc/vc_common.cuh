@@ -21,6 +21,7 @@ struct Req {                 // one request of a batch
   int64_t out_row0;          // first output row (K_out/V_out/idx_out)
   int64_t drop_row0;         // first drop-list row
   int64_t lsep_off;          // float offset of its chunk-padded row normalisers [L][Hkv][C*128]
+  int64_t vs_row0;           // first row of its compacted survivors' values (tensor-core fusion)
   int32_t n, W, Nq, h;
   int32_t C;                 // 128-row chunks of one (layer, KV head) row set, ceil(G*W/128)
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
@@ -51,7 +52,8 @@ struct Tables {              // device pointers into the workspace
   const int64_t* row0_out;   // [n_req * L + 1] first output row of each (request, layer)
   const int32_t* unit0_tc1;  // [n_req + 1] CTAs of the tensor-core lse pass
   const int32_t* unit0_tc2;  // [n_req + 1] CTAs of the tensor-core column-sum pass
-  const int32_t* unit0_fuse_tc;  // [n_req * L + 1] 128-row kept tiles x Hkv (tensor-core fusion)
+  const int32_t* unit0_fuse_tc;  // [n_req * L + 1] 256-row kept tiles x Hkv (tensor-core fusion)
+  const int32_t* unit0_gather;   // [n_req * L + 1] 16-row survivor blocks x Hkv (row gather)
   int32_t* status;           // device status word
 };
 

@@ -80,7 +80,7 @@ def lib() -> ctypes.CDLL:
         L.prunekv_select_workspace_size.argtypes = [i32, i32, i32, i32]
         L.prunekv_select_workspace_size.restype = sz
         L.prunekv_select.argtypes = [vp, i32, i32, i32, pi32, i32, i32, vp, vp, vp, vp, sz, vp]
-        L.prunekv_fuse_workspace_size.argtypes = [i32]
+        L.prunekv_fuse_workspace_size.argtypes = [pi32, i32, i32, i32, i32, i32]
         L.prunekv_fuse_workspace_size.restype = sz
         L.prunekv_fuse_compact.argtypes = [vp, vp, i32, i32, i32, i32, i32, pi32, i32, vp, vp, f32,
                                            f32, vp, vp, vp, sz, vp]
@@ -217,8 +217,8 @@ def prunekv_select(scores: torch.Tensor, B: Sequence[int], Nq: int, rank_mode: i
     return rank, keep[:Hkv * sum(B)], drop[:drop_rows(B, Nq, Hkv)]
 
 
-def prunekv_fuse_workspace_size(L: int) -> int:
-    return lib().prunekv_fuse_workspace_size(L)
+def prunekv_fuse_workspace_size(B: Sequence[int], Hkv: int, d: int, n_vis: int, Nq: int) -> int:
+    return lib().prunekv_fuse_workspace_size(_i32(B), len(B), Hkv, d, n_vis, Nq)
 
 
 def prunekv_fuse_compact(K: torch.Tensor, V: torch.Tensor, B: Sequence[int], Nq: int,
@@ -235,7 +235,7 @@ def prunekv_fuse_compact(K: torch.Tensor, V: torch.Tensor, B: Sequence[int], Nq:
         V_out = torch.empty((max(rows, 1), d), dtype=V.dtype, device=V.device)
     keep_idx = keep_idx if keep_idx.numel() else torch.zeros(1, dtype=torch.int32, device=K.device)
     drop_idx = drop_idx if drop_idx.numel() else torch.zeros(1, dtype=torch.int32, device=K.device)
-    ws = _workspace(prunekv_fuse_workspace_size(L), K.device, ws)
+    ws = _workspace(prunekv_fuse_workspace_size(B, Hkv, d, n, Nq), K.device, ws)
     _check("prunekv_fuse_compact", lib().prunekv_fuse_compact(
         _ptr(K), _ptr(V), _dtype_code(K), L, Hkv, d, n, _i32(B), Nq, _ptr(keep_idx),
         _ptr(drop_idx), float(mu), float(tau), _ptr(K_out), _ptr(V_out), _ptr(ws), ws.numel(),

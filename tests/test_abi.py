@@ -93,7 +93,7 @@ def test_workspace_sizes_are_positive_and_aligned():
     assert vc.prunekv_score_workspace_size(28, 28, 64) % 256 == 0
     assert vc.prunekv_score_workspace_size(28, 28, 64) >= 28 * 28 * 64 * 4
     assert vc.prunekv_select_workspace_size(28, 4, 12544) >= 2 * 8 * 4 * 12544
-    assert vc.prunekv_fuse_workspace_size(28) > 0
+    assert vc.prunekv_fuse_workspace_size([3833, 1916], 4, 128, 12544, 4237) > 4 * 4237 * 2 * 256
     b = vc.Batch([12544], [64], [(19, 100)])
     prm = vc.make_params(28, 28, 4, 128, vc.VC_BF16)
     assert vc.prunekv_workspace_size(b, prm) > vc.prunekv_score_workspace_size(28, 28, 64)

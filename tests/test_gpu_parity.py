@@ -149,7 +149,7 @@ def test_bad_index_sets_device_status():
     B, Nq = [4], 6
     keep = torch.tensor([1, 2, 3, 999], dtype=torch.int32, device=DEV)
     drop = torch.tensor([5, 6], dtype=torch.int32, device=DEV)
-    ws = torch.empty(vc.prunekv_fuse_workspace_size(L), dtype=torch.uint8, device=DEV)
+    ws = torch.empty(vc.prunekv_fuse_workspace_size(B, Hkv, d, n, Nq), dtype=torch.uint8, device=DEV)
     vc.prunekv_fuse_compact(K, V, B, Nq, keep, drop, ws=ws)
     assert vc.prunekv_get_status(ws) == vc.VC_ERR_DEVICE_INDEX
     keep[3] = 4

@@ -56,6 +56,7 @@ struct Layout {
   std::vector<int32_t> u_tc1, u_tc2, base_tc1, u_fuse_tc, u_gather;
   int units_fuse_tc = 0, units_gather = 0;
   int64_t vs_rows = 0;
+  int max_n = 0;
   // derived sizes
   int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
   int units_lse = 0, units_col = 0, units_fuse = 0;
@@ -82,6 +83,7 @@ struct Layout {
     u_fuse_tc.assign((size_t)n_req * L + 1, 0);
     u_gather.assign((size_t)n_req * L + 1, 0);
     vs_rows = 0;
+    max_n = 0;
     u_tc2.assign(n_req + 1, 0);
     base_tc1.assign(n_req, 0);
     q_rows = k_rows = max_rows = prows = max_prows = 0;
@@ -104,6 +106,7 @@ struct Layout {
       q.C = (G * p.W + 127) / 128;
       q.lsep_off = prows;
       q.vs_row0 = vs_rows;
+      max_n = std::max(max_n, p.n);
       prows += (int64_t)L * Hkv * q.C * 128;
       max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
       q.nrb = (G * p.W + 255) / 256;
@@ -443,7 +446,7 @@ int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis, c
   cudaError_t e = lay.upload(w, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
   const int problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
-  e = launch_select(lay.shape(1.f), lay.tables(w), problems, scores, rank_out,
+  e = launch_select(lay.shape(1.f), lay.tables(w), problems, lay.max_n, scores, rank_out,
                     reinterpret_cast<uint32_t*>(w + lay.o_keys),
                     reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, keep_idx,
                     drop_idx, st);
@@ -508,7 +511,7 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   const Shape sh = lay.shape(scale);
   const Tables tb = lay.tables(w);
   const int problems = lay.n_req * (p->rank_mode == VC_RANK_PER_LAYER ? p->L * p->Hkv : p->Hkv);
-  e = launch_select(sh, tb, problems, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
+  e = launch_select(sh, tb, problems, lay.max_n, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
                     reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
   e = launch_fuse(p->dtype, K, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, K_out, V_out, w, st);

@@ -49,9 +49,10 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
                            int units, cudaStream_t st);
 
 // Ranking (radix sort per problem) and ascending keep/drop compaction.
-cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, const float* scores,
-                          int32_t* rank, uint32_t* keys, int32_t* vals, int64_t sort_stride,
-                          int32_t* keep_idx, int32_t* drop_idx, cudaStream_t st);
+cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int max_n,
+                          const float* scores, int32_t* rank, uint32_t* keys, int32_t* vals,
+                          int64_t sort_stride, int32_t* keep_idx, int32_t* drop_idx,
+                          cudaStream_t st);
 
 // K_out = K[keep] (bit-exact), total_rows = Hkv * sum over requests and layers of B_l.
 cudaError_t launch_gather_k(int dtype, const void* K, const Shape& sh, const Tables& tb,

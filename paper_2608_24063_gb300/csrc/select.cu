@@ -22,6 +22,20 @@ namespace {
 constexpr int kSortThreads = 1024;
 constexpr int kSortWarps = kSortThreads / 32;
 
+// Lanes of the warp holding the same 8-bit digit (and the same validity),
+// built from nine ballots.
+__device__ __forceinline__ uint32_t digit_peers(uint32_t dig, bool ok) {
+  const uint32_t okm = __ballot_sync(0xffffffffu, ok);
+  uint32_t peers = ok ? okm : ~okm;
+#pragma unroll
+  for (int b = 0; b < 8; ++b) {
+    const uint32_t bit = (dig >> b) & 1u;
+    const uint32_t m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
+  }
+  return peers;
+}
+
 __device__ __forceinline__ uint32_t desc_key(float s) {
   // monotone map float -> uint32 (ascending), then invert for descending order
   uint32_t u = __float_as_uint(s);
@@ -87,7 +101,7 @@ __global__ void __launch_bounds__(kSortThreads) rank_sort_kernel(Shape sh, Table
       const int e = s0 + c + lane;
       const bool ok = e < n;
       const uint32_t dig = ok ? (kin[e] >> shift) & 0xffu : 0x100u + lane;
-      const uint32_t peers = __match_any_sync(0xffffffffu, dig);
+      const uint32_t peers = digit_peers(dig, ok);
       if (ok && (peers & lt_mask) == 0) hist[warp][dig] += __popc(peers);
       __syncwarp();
     }
@@ -126,7 +140,7 @@ __global__ void __launch_bounds__(kSortThreads) rank_sort_kernel(Shape sh, Table
       const bool ok = e < n;
       const uint32_t key = ok ? kin[e] : 0u;
       const uint32_t dig = ok ? (key >> shift) & 0xffu : 0x100u + lane;
-      const uint32_t peers = __match_any_sync(0xffffffffu, dig);
+      const uint32_t peers = digit_peers(dig, ok);
       uint32_t pos = 0;
       if (ok) pos = digit_base[dig] + hist[warp][dig] + __popc(peers & lt_mask);
       __syncwarp();
@@ -146,6 +160,99 @@ __global__ void __launch_bounds__(kSortThreads) rank_sort_kernel(Shape sh, Table
     const int v = vin[e];
     if (v >= 0 && v < n) p.rank[v] = e;
   }
+}
+
+// Shared-memory variant for n <= kSmemSortMax: keys, token ids and the
+// per-warp histograms stay on chip; only the scores are read and the ranks
+// written.  Same stable LSD passes as rank_sort_kernel.
+constexpr int kSmemSortMax = 16384;
+
+__global__ void __launch_bounds__(kSortThreads) rank_sort_smem_kernel(Shape sh, Tables tb,
+                                                                      const float* __restrict__ scores,
+                                                                      int32_t* __restrict__ rank) {
+  extern __shared__ uint4 smem_u4[];
+  uint32_t* k0 = reinterpret_cast<uint32_t*>(smem_u4);
+  uint32_t* k1 = k0 + kSmemSortMax;
+  uint16_t* v0 = reinterpret_cast<uint16_t*>(k1 + kSmemSortMax);
+  uint16_t* v1 = v0 + kSmemSortMax;
+  uint16_t (*hist)[256] = reinterpret_cast<uint16_t (*)[256]>(v1 + kSmemSortMax);
+  __shared__ uint32_t digit_base[256];
+  const int per_req = sh.rank_mode == VC_RANK_PER_LAYER ? sh.L * sh.Hkv : sh.Hkv;
+  const int r = blockIdx.x / per_req, kprob = blockIdx.x % per_req;
+  const Req rq = tb.req[r];
+  const int64_t off = rq.s_off + (int64_t)kprob * rq.n;
+  const int n = rq.n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  const int seg = ((n + kSortWarps * 32 - 1) / (kSortWarps * 32)) * 32;
+  const int s0 = warp * seg;
+  for (int e = threadIdx.x; e < n; e += kSortThreads) {
+    k0[e] = desc_key(scores[off + e]);
+    v0[e] = (uint16_t)e;
+  }
+  uint32_t* kin = k0; uint32_t* kout = k1;
+  uint16_t* vin = v0; uint16_t* vout = v1;
+  __syncthreads();
+  for (int shift = 0; shift < 32; shift += 8) {
+    for (int d = lane; d < 256; d += 32) hist[warp][d] = 0;
+    __syncwarp();
+    for (int c = 0; c < seg; c += 32) {
+      const int e = s0 + c + lane;
+      const bool ok = e < n;
+      const uint32_t dig = ok ? (kin[e] >> shift) & 0xffu : 0x100u + lane;
+      const uint32_t peers = digit_peers(dig, ok);
+      if (ok && (peers & lt_mask) == 0) hist[warp][dig] += (uint16_t)__popc(peers);
+      __syncwarp();
+    }
+    __syncthreads();
+    if (threadIdx.x < 256) {
+      const int d = threadIdx.x;
+      uint32_t run = 0;
+      for (int w = 0; w < kSortWarps; ++w) {
+        const uint32_t cnt = hist[w][d];
+        hist[w][d] = (uint16_t)run;
+        run += cnt;
+      }
+      digit_base[d] = run;
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      uint32_t v[8], sum = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { v[i] = digit_base[lane * 8 + i]; sum += v[i]; }
+      uint32_t incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      uint32_t run = incl - sum;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) { digit_base[lane * 8 + i] = run; run += v[i]; }
+    }
+    __syncthreads();
+    for (int c = 0; c < seg; c += 32) {
+      const int e = s0 + c + lane;
+      const bool ok = e < n;
+      const uint32_t key = ok ? kin[e] : 0u;
+      const uint32_t dig = ok ? (key >> shift) & 0xffu : 0x100u + lane;
+      const uint32_t peers = digit_peers(dig, ok);
+      uint32_t pos = 0;
+      if (ok) pos = digit_base[dig] + hist[warp][dig] + __popc(peers & lt_mask);
+      __syncwarp();
+      if (ok && (peers & lt_mask) == 0) hist[warp][dig] += (uint16_t)__popc(peers);
+      if (ok) {
+        if (pos < (uint32_t)n) { kout[pos] = key; vout[pos] = vin[e]; }
+        else set_status(tb.status, VC_ERR_DEVICE_INDEX);
+      }
+      __syncwarp();
+    }
+    __syncthreads();
+    uint32_t* tk = kin; kin = kout; kout = tk;
+    uint16_t* tv = vin; vin = vout; vout = tv;
+  }
+  int32_t* rk = rank + off;
+  for (int e = threadIdx.x; e < n; e += kSortThreads) rk[vin[e]] = e;
 }
 
 // One CTA per (request, layer, KV head); layers with B_l == 0 exit at once.
@@ -216,10 +323,18 @@ __global__ void __launch_bounds__(kScanThreads) compact_kernel(Shape sh, Tables 
 
 }  // namespace
 
-cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, const float* scores,
-                          int32_t* rank, uint32_t* keys, int32_t* vals, int64_t sort_stride,
-                          int32_t* keep_idx, int32_t* drop_idx, cudaStream_t st) {
-  {
+cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int max_n,
+                          const float* scores, int32_t* rank, uint32_t* keys, int32_t* vals,
+                          int64_t sort_stride, int32_t* keep_idx, int32_t* drop_idx,
+                          cudaStream_t st) {
+  if (max_n <= kSmemSortMax) {
+    const size_t smem = (size_t)kSmemSortMax * (2 * 4 + 2 * 2) + (size_t)kSortWarps * 256 * 2;
+    cudaError_t e = cudaFuncSetAttribute(rank_sort_smem_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    ProfileScope ps("rank_sort", st);
+    rank_sort_smem_kernel<<<n_problems, kSortThreads, smem, st>>>(sh, tb, scores, rank);
+  } else {
     ProfileScope ps("rank_sort", st);
     rank_sort_kernel<<<n_problems, kSortThreads, 0, st>>>(sh, tb, scores, rank, keys, vals,
                                                           sort_stride);

@@ -269,3 +269,29 @@ def test_generator_same_bits_on_device():
     k_cpu, v_cpu = synth.make_kv(wl, 0, q_cpu, "cpu", layers=[1])
     k_dev, v_dev = synth.make_kv(wl, 0, q_cpu, DEV, layers=[1])
     assert torch.equal(k_cpu[1], k_dev[1].cpu()) and torch.equal(v_cpu[1], v_dev[1].cpu())
+
+
+@pytest.mark.parametrize("n", [1, 31, 1025, 16384, 16385, 32768])
+@pytest.mark.parametrize("mode", [vc.VC_RANK_SHARED, vc.VC_RANK_PER_LAYER], ids=["shared", "layer"])
+def test_select_matches_oracle_ranking(n, mode):
+    # shared-memory sort up to 16384 tokens, global-memory sort beyond; exact ties
+    # (scores drawn from a small set) must go to the lower index.
+    L, Hkv = 3, 2
+    rng = np.random.default_rng(n + 7 * mode)
+    shape = (Hkv, n) if mode == vc.VC_RANK_SHARED else (L, Hkv, n)
+    s = rng.integers(0, max(2, n // 3), size=shape).astype(np.float32) / 7.0
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 1, 3)
+    rank, keep, drop = vc.prunekv_select(torch.from_numpy(s).to(DEV), B, Nq, mode)
+    torch.cuda.synchronize()
+    keep_ref, drop_ref, rank_ref = ok.select(s.astype(np.float64), B, Nq,
+                                             "per_layer" if mode else "shared")
+    assert np.array_equal(rank.cpu().numpy(), rank_ref)
+    keep, drop = keep.cpu().numpy(), drop.cpu().numpy()
+    P = Qd = 0
+    for l in range(L):
+        D = Nq - B[l] if B[l] > 0 else 0
+        for g in range(Hkv):
+            assert np.array_equal(keep[Hkv * P + g * B[l]:Hkv * P + (g + 1) * B[l]], keep_ref[l][g])
+            assert np.array_equal(drop[Hkv * Qd + g * D:Hkv * Qd + (g + 1) * D], drop_ref[l][g])
+        P += B[l]
+        Qd += D

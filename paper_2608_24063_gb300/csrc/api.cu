@@ -179,19 +179,20 @@ struct Layout {
   }
 
   // Key splits of the tensor-core lse pass: pick S in [1, max] that fills the
-  // last wave of CTAs best (one CTA per SM); ties go to the smaller S.
+  // last wave of CTA pairs best (`slots` pairs resident at once); ties go to
+  // the smaller S.
   void set_splits(int s) {
     S = s;
     for (int r = 0; r < n_req; ++r) u_tc1[r + 1] = u_tc1[r] + base_tc1[r] * S;
   }
-  void choose_splits(int nsm) {
+  void choose_splits(int slots) {
     int best = 1;
     double best_eff = -1.0;
     for (int s = 1; s <= score_tc_max_splits(); ++s) {
       int64_t units = 0;
       for (int r = 0; r < n_req; ++r) units += (int64_t)base_tc1[r] * s;
-      const int64_t waves = (units + nsm - 1) / nsm;
-      const double eff = (double)units / (double)(waves * nsm);
+      const int64_t waves = (units + slots - 1) / slots;
+      const double eff = (double)units / (double)(waves * slots);
       if (eff > best_eff + 1e-9) { best_eff = eff; best = s; }
     }
     set_splits(best);
@@ -275,7 +276,7 @@ struct Layout {
 cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, float scale,
                          uint8_t* w, const float* row_lse, float* scores, cudaStream_t st) {
   const bool tc = g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128;
-  if (tc) lay.choose_splits(sm_count());
+  if (tc) lay.choose_splits(score_tc_pair_slots());
   cudaError_t e = lay.upload(w, st);
   if (e != cudaSuccess) return e;
   const Shape sh = lay.shape(scale);

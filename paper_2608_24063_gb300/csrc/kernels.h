@@ -26,7 +26,7 @@ cudaError_t launch_score_simt(int dtype, const void* Qw, const void* K, const Sh
 // Eq. (token_score) on tcgen05 tensor cores (bf16, d = 128): lse pass (skipped when
 // lse_nat != nullptr), merge of key splits, column sums.
 struct TcPlan {
-  int units1;        // CTAs of the lse pass (sum over requests of L*Hkv*nrb*S)
+  int units1;        // CTA pairs of the lse pass (sum over requests of L*Hkv*nrb*S)
   int units2;        // CTAs of the column-sum pass (sum of Hkv*tiles)
   int S;             // key splits of the lse pass
   int64_t q_rows;    // rows of the packed Qw tensor
@@ -35,6 +35,7 @@ struct TcPlan {
   int64_t max_prows; // max over requests of L*Hkv*C*128 (chunk-padded rows)
 };
 int score_tc_max_splits();
+int score_tc_pair_slots();
 cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
                             const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
                             float* scores, cudaStream_t st);

@@ -6,9 +6,9 @@
 // swizzling.  The exact softmax column sum needs every row's normaliser
 // first, so the score takes two passes over the logits:
 //
-//   pass 1 (score_lse_tc)    rows in TMEM lanes: per row, running max and
-//                            compensated sum of exp2 over a range of key
-//                            tiles -> partial (m, z) per key split;
+//   pass 1 (score_lse_tc)    CTA pairs, rows in TMEM lanes: per row, running
+//                            max and compensated sum of exp2 over a range of
+//                            256-key tiles -> partial (m, z) per key split;
 //   merge  (lse_merge)       -lse2 = -(m + log2 z) over the splits (or minus
 //                            the caller's natural-log normaliser * log2 e),
 //                            written per (layer, KV head) in 128-row chunks
@@ -21,13 +21,17 @@
 //
 // Warp roles in both passes (320 threads, one CTA per SM): warps 0-3 and 4-7
 // are two consumer warpgroups (one TMEM lane per thread), warp 8 issues TMA and
-// owns the tensor-memory allocation, one thread of warp 9 issues the MMAs.
+// owns the tensor-memory allocation, one thread of warp 9 issues the MMAs (in
+// pass 1 only the even CTA of each pair issues them, as 2-SM MMAs: M = 256
+// rows, N = 256 keys, 128 cycles each, so the issuing thread's barrier waits
+// and commits hide behind the tensor pipe).
 // Each consumer thread takes a whole tile (up to 128 accumulators) per step,
 // so its exps and sums form many independent chains.  Every wait is bounded: on a
 // timeout the CTA stops issuing, waits for its own copies and MMAs, frees its
 // tensor memory and records VC_ERR_DEVICE_TIMEOUT.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "kernels.h"
@@ -85,182 +89,220 @@ __device__ __forceinline__ float exp2_sum16(const float (&x)[16], float2 s, cons
 }
 
 // ---------------------------------------------------------------------------
-// pass 1
+// pass 1 on CTA pairs
+//
+// A pair covers 256 window rows (128 per CTA, rows in TMEM lanes) and walks
+// its key range in tiles of 256 keys: each CTA loads its 128 query rows once
+// and, per tile, its own 128 keys (CTA r: keys r*128 ... r*128+127 of the
+// tile); one 2-SM MMA chain (M = 256, N = 256, K = 128) leaves every row's 256
+// logits in its own CTA's tensor memory.  Tensor memory: 2 slots x 256
+// columns; consumer warpgroup wg drains slot wg (tiles i with i % 2 == wg),
+// so the MMA fills one slot while the other is read, and the two warpgroups'
+// per-row (max, sum) pairs are merged at the end.
+
+constexpr uint32_t kPairKeys = 256;             // keys per pass-1 tile (both CTAs)
+constexpr int kStagesPair = 4;                  // K ring of pass 1 (per CTA: 32 KB a stage)
 
 struct P1Smem {
-  uint8_t q[2][2][kKBlockBytes];          // [row block][K-block]
-  uint8_t k[kStages1][2][kKBlockBytes];   // [stage][K-block]
-  uint64_t q_full;
-  uint64_t k_full[kStages1], k_empty[kStages1];
-  uint64_t tm_full[2][2], tm_empty[2][2]; // [row block][slot]
+  uint8_t q[2][kKBlockBytes];               // this CTA's 128 query rows [K-block]
+  uint8_t k[kStagesPair][2][kKBlockBytes];  // this CTA's 128 keys of the tile [stage][K-block]
+  float2 half[4][32];                       // (max, sum) of warpgroup 1, merged at the end
+  uint64_t q_full;                          // even CTA: both CTAs' Q rows landed
+  uint64_t k_full[kStagesPair];             // even CTA: both CTAs' key halves landed
+  uint64_t k_empty[kStagesPair];            // both: the MMAs reading the stage are done
+  uint64_t tm_full[2];                      // both: the slot's logits are ready
+  uint64_t tm_empty[2];                     // even CTA: the slot's 8 consumer warps copied it out
   uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
 };
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     Shape sh, Tables tb, int S, float2* __restrict__ part) {
   extern __shared__ uint8_t smem_raw[];
   P1Smem& sm = *reinterpret_cast<P1Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int unit = (int)(blockIdx.x >> 1);
 
-  const int r = upper_index(tb.unit0_tc1, sh.n_req, (int32_t)blockIdx.x);
+  const int r = upper_index(tb.unit0_tc1, sh.n_req, (int32_t)unit);
   const Req rq = tb.req[r];
-  int u = blockIdx.x - tb.unit0_tc1[r];
+  int u = unit - tb.unit0_tc1[r];
   const int s = u % S;
   u /= S;
   const int rbp = u % rq.nrb;
   u /= rq.nrb;
   const int g = u % sh.Hkv, l = u / sh.Hkv;
   const int rows = sh.G * rq.W;
-  const int nblk = (rows - rbp * 256) > (int)kTile ? 2 : 1;   // row blocks with valid rows
-  const int tps = (rq.tiles + S - 1) / S;
+  const int ntiles_all = (rq.n + (int)kPairKeys - 1) / (int)kPairKeys;
+  const int tps = (ntiles_all + S - 1) / S;
   const int t_begin = s * tps;
-  const int ntiles = max(0, min(rq.tiles, t_begin + tps) - t_begin);
-  const int qrow0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + rbp * 256;
-  const int krow0 = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n);
+  const int ntiles = max(0, min(ntiles_all, t_begin + tps) - t_begin);
+  const int qrow = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + rbp * 256 +
+                   (int)rank * (int)kTile;
+  const int krow0 = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + (int)rank * (int)kTile;
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
-    for (int i = 0; i < kStages1; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
-    for (int b = 0; b < 2; ++b)
-      for (int i = 0; i < 2; ++i) { mbar_init(&sm.tm_full[b][i], 1); mbar_init(&sm.tm_empty[b][i], kTile); }
+    for (int i = 0; i < kStagesPair; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
+    for (int i = 0; i < 2; ++i) { mbar_init(&sm.tm_full[i], 1); mbar_init(&sm.tm_empty[i], 8); }
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (warp == kProducerWarp) {
-    tmem_alloc(&sm.tmem_base, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, kTmemCols);
+    tmem_relinquish_pair();
   }
+  __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();                  // barriers of both CTAs initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
   if (warp == kProducerWarp && lane == 0) {
-    // ---- TMA producer
+    // ---- TMA producer (both CTAs): own rows and key halves, counted on the even CTA's barriers
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
-    mbar_arrive_expect_tx(&sm.q_full, nblk * kTileBytes);
-    for (int b = 0; b < nblk; ++b)
-      for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.q[b][kb], &tmQ, kb * 64, qrow0 + b * (int)kTile, &sm.q_full);
+    const uint32_t q_full0 = map_to_rank(smem_u32(&sm.q_full), 0);
+    if (rank == 0) mbar_arrive_expect_tx(&sm.q_full, 2 * kTileBytes);
+    for (int kb = 0; kb < 2; ++kb) tma_load_2d_pair(sm.q[kb], &tmQ, kb * 64, qrow, q_full0);
     int issued = 0;
     for (int i = 0; i < ntiles; ++i) {
-      const int st = i % kStages1;
-      if (!mbar_wait(&sm.k_empty[st], ((i / kStages1) & 1) ^ 1, abort)) break;
-      mbar_arrive_expect_tx(&sm.k_full[st], kTileBytes);
-      const int y = krow0 + (t_begin + i) * (int)kTile;
-      tma_load_2d(sm.k[st][0], &tmK, 0, y, &sm.k_full[st]);
-      tma_load_2d(sm.k[st][1], &tmK, 64, y, &sm.k_full[st]);
+      const int st = i % kStagesPair;
+      if (!mbar_wait(&sm.k_empty[st], ((i / kStagesPair) & 1) ^ 1, abort)) break;
+      if (rank == 0) mbar_arrive_expect_tx(&sm.k_full[st], 2 * kTileBytes);
+      const uint32_t k_full0 = map_to_rank(smem_u32(&sm.k_full[st]), 0);
+      const int y = krow0 + (t_begin + i) * (int)kPairKeys;
+      tma_load_2d_pair(sm.k[st][0], &tmK, 0, y, k_full0);
+      tma_load_2d_pair(sm.k[st][1], &tmK, 64, y, k_full0);
       ++issued;
     }
-    // every copy this CTA started has landed before the CTA may exit
-    drain_wait(&sm.q_full, 0);
-    for (int i = max(0, issued - kStages1); i < issued; ++i)
-      drain_wait(&sm.k_full[i % kStages1], (i / kStages1) & 1);
-  } else if (warp == kMmaWarp && lane == 0) {
-    // ---- MMA issuer
-    const uint32_t idesc = idesc_bf16_f32(kTile, kTile);
+    // the even CTA waits until every copy of both CTAs has landed
+    if (rank == 0) {
+      drain_wait(&sm.q_full, 0);
+      for (int i = max(0, issued - kStagesPair); i < issued; ++i)
+        drain_wait(&sm.k_full[i % kStagesPair], (i / kStagesPair) & 1);
+    }
+  } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
+    // ---- MMA issuer (even CTA): D[row][key] for 256 rows x 256 keys per tile
+    const uint32_t idesc = idesc_bf16_f32(2 * kTile, kPairKeys);
     bool ok = mbar_wait(&sm.q_full, 0, abort);
     for (int i = 0; ok && i < ntiles; ++i) {
-      const int st = i % kStages1;
-      if (!mbar_wait(&sm.k_full[st], (i / kStages1) & 1, abort)) break;
-      tc_fence_after();
+      const int st = i % kStagesPair;
       const int slot = i & 1;
-      const uint32_t use = (uint32_t)i >> 1;
-      for (int b = 0; b < nblk && ok; ++b) {
-        if (!mbar_wait(&sm.tm_empty[b][slot], (use & 1) ^ 1, abort)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t d = tbase + (uint32_t)(b * 2 + slot) * kTile;
+      if (!mbar_wait(&sm.k_full[st], (i / kStagesPair) & 1, abort)) break;
+      if (!mbar_wait(&sm.tm_empty[slot], ((i >> 1) & 1) ^ 1, abort)) break;
+      tc_fence_after();
+      const uint32_t d = tbase + (uint32_t)slot * kPairKeys;
 #pragma unroll
-        for (int kb = 0; kb < 2; ++kb)
+      for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            mma_bf16(d, desc_sw128(smem_u32(sm.q[b][kb]) + k * 32),
-                     desc_sw128(smem_u32(sm.k[st][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
-        mma_commit(&sm.tm_full[b][slot]);
-      }
-      if (ok) mma_commit(&sm.k_empty[st]);
+        for (int k = 0; k < 4; ++k)
+          mma_bf16_pair(d, desc_sw128(smem_u32(sm.q[kb]) + k * 32),
+                        desc_sw128(smem_u32(sm.k[st][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
+      mma_commit_pair(&sm.tm_full[slot], 3);
+      mma_commit_pair(&sm.k_empty[st], 3);
     }
-    mma_commit(&sm.mma_done);
+    mma_commit_pair(&sm.mma_done, 1);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
-    // ---- row statistics: one thread per row (= TMEM lane)
-    const int b = warp >> 2;
+    // ---- row statistics: one thread per row (= TMEM lane).  Warpgroup wg
+    // takes the tiles i with i % 2 == wg (TMEM slot wg), all 256 columns in
+    // two halves, so the two warpgroups on a sub-partition run a tile apart
+    // and one's waits and TMEM loads overlap the other's exps.
+    const int wg = warp >> 2;
     const int lrow = ((warp & 3) << 5) + lane;
     const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    const uint32_t tm_empty0 = lane == 0 ? map_to_rank(smem_u32(&sm.tm_empty[wg]), 0) : 0u;
     const float s2 = sh.scale_log2;
     float m = -INFINITY;
     Kahan z;
     z.init();
-    for (int i = 0; b < nblk && i < ntiles; ++i) {
-      const int slot = i & 1;
-      const uint32_t use = (uint32_t)i >> 1;
-      if (!warp_wait(&sm.tm_full[b][slot], use & 1, abort)) break;
+    for (int i = wg; i < ntiles; i += 2) {
+      if (!warp_wait(&sm.tm_full[wg], (i >> 1) & 1, abort)) break;
       tc_fence_after();
-      const int valid = min((int)kTile, rq.n - (t_begin + i) * (int)kTile);
-      const uint32_t col0 = tbase + lane_off + (uint32_t)(b * 2 + slot) * kTile;
-      float x[8][16];
-      {
-        uint32_t v[8][16];
+#pragma unroll 1
+      for (int hf = 0; hf < 2; ++hf) {
+        const int valid = min((int)kTile, rq.n - (t_begin + i) * (int)kPairKeys - hf * (int)kTile);
+        const uint32_t col0 = tbase + lane_off + (uint32_t)wg * kPairKeys + (uint32_t)hf * kTile;
+        float x[8][16];
+        {
+          uint32_t v[8][16];
 #pragma unroll
-        for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, v[p]);
-        tmem_wait_only();
+          for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, v[p]);
+          tmem_wait_only();
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {
+            reg_fence(v[p]);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
+          }
+        }
+        if (hf == 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(tm_empty0);   // slot copied out
+        }
+        if (valid < (int)kTile) {                 // keys >= n (ragged last tile)
+#pragma unroll
+          for (int p = 0; p < 8; ++p)
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              if (p * 16 + j >= valid) x[p][j] = -INFINITY;
+        }
+        float pm[8];
 #pragma unroll
         for (int p = 0; p < 8; ++p) {
-          reg_fence(v[p]);
+          float a = fmaxf(x[p][0], x[p][1]);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
+          for (int j = 2; j < 16; j += 2) a = fmax3(a, x[p][j], x[p][j + 1]);
+          pm[p] = a;
+        }
+        const float cm = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
+        const float xm = cm * s2;
+        if (xm > m) {
+          const float c = ex2(m - xm);
+          z.s *= c;
+          z.c *= c;
+          m = xm;
+        }
+        if (m != -INFINITY) {
+          float2 nb[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) nb[j] = make_float2(-m, -m);
+          float ps[8];
+#pragma unroll
+          for (int p = 0; p < 8; ++p) ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
+          z.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
         }
       }
-      tc_fence_before();
-      mbar_arrive(&sm.tm_empty[b][slot]);       // columns copied out: the MMA may reuse them
-      if (valid < (int)kTile) {                 // last tile of the request: mask keys >= n
-#pragma unroll
-        for (int p = 0; p < 8; ++p)
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (p * 16 + j >= valid) x[p][j] = -INFINITY;
-      }
-      float pm[8];
-#pragma unroll
-      for (int p = 0; p < 8; ++p) {
-        float a = fmaxf(x[p][0], x[p][1]);
-#pragma unroll
-        for (int j = 2; j < 16; j += 2) a = fmax3(a, x[p][j], x[p][j + 1]);
-        pm[p] = a;
-      }
-      const float cm = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
-      const float xm = cm * s2;
-      if (xm > m) {
-        const float c = ex2(m - xm);
-        z.s *= c;
-        z.c *= c;
-        m = xm;
-      }
-      if (m != -INFINITY) {
-        float2 nb[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) nb[j] = make_float2(-m, -m);
-        float ps[8];
-#pragma unroll
-        for (int p = 0; p < 8; ++p) ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
-        z.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
-      }
     }
-    const int rho = rbp * 256 + b * (int)kTile + lrow;
-    if (rho < rows)
-      part[(rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho) * S + s] = make_float2(m, z.s);
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == kProducerWarp) {
+    // merge the two warpgroups' statistics of each row
+    if (wg == 1) sm.half[warp & 3][lane] = make_float2(m, z.s);
     __syncwarp();
+    named_sync(1, 256);
+    if (wg == 0) {
+      const float2 o = sm.half[warp & 3][lane];
+      const float mm = fmaxf(m, o.x);
+      float zz = 0.f;
+      if (mm != -INFINITY) {
+        if (m != -INFINITY) zz += z.s * ex2(m - mm);
+        if (o.x != -INFINITY) zz += o.y * ex2(o.x - mm);
+      }
+      const int rho = rbp * 256 + (int)rank * (int)kTile + lrow;
+      if (rho < rows)
+        part[(rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho) * S + s] = make_float2(mm, zz);
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync();                  // no CTA leaves while the pair's MMAs or copies may touch it
+  if (warp == kProducerWarp) {
     tc_fence_after();
-    tmem_dealloc(tbase, kTmemCols);
+    tmem_dealloc_pair(tbase, kTmemCols);
   }
   if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
 }
@@ -526,7 +568,33 @@ bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows) {
 
 }  // namespace
 
-int score_tc_max_splits() { return 2; }
+int score_tc_max_splits() { return 4; }
+
+// CTA pairs of the lse pass that fit on the device at once (pairs must sit on
+// one TPC, so this can be below half the SM count).
+int score_tc_pair_slots() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (cached[dev] > 0) return cached[dev];
+  const size_t smem1 = sizeof(P1Smem) + 1024;
+  if (cudaFuncSetAttribute(score_lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1) !=
+      cudaSuccess)
+    return 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, score_lse_tc_kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    int sms = 2;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    n = std::max(1, sms / 2);
+  }
+  cached[dev] = n;
+  return n;
+}
 
 cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, const Tables& tb,
                             const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
@@ -540,7 +608,7 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
     e = cudaFuncSetAttribute(score_lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
     if (e != cudaSuccess) return e;
     ProfileScope ps("score_lse_tc", st);
-    score_lse_tc_kernel<<<tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part);
+    score_lse_tc_kernel<<<2 * tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

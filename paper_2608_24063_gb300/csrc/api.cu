@@ -103,14 +103,14 @@ struct Layout {
       q.out_row0 = out_rows;
       q.drop_row0 = drop_rows;
       q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
-      q.C = (G * p.W + 127) / 128;
+      q.C = 2 * ((G * p.W + 255) / 256);
       q.lsep_off = prows;
       q.vs_row0 = vs_rows;
       max_n = std::max(max_n, p.n);
       prows += (int64_t)L * Hkv * q.C * 128;
       max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
       q.nrb = (G * p.W + 255) / 256;
-      q.tiles = (p.n + 127) / 128;
+      q.tiles = (p.n + 255) / 256;
       base_tc1[r] = L * Hkv * q.nrb;
       u_tc2[r + 1] = u_tc2[r] + Hkv * q.tiles;
       q_rows += (int64_t)L * Hq * p.W;

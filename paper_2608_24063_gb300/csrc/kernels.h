@@ -27,7 +27,7 @@ cudaError_t launch_score_simt(int dtype, const void* Qw, const void* K, const Sh
 // lse_nat != nullptr), merge of key splits, column sums.
 struct TcPlan {
   int units1;        // CTA pairs of the lse pass (sum over requests of L*Hkv*nrb*S)
-  int units2;        // CTAs of the column-sum pass (sum of Hkv*tiles)
+  int units2;        // CTA pairs of the column-sum pass (sum of Hkv*tiles)
   int S;             // key splits of the lse pass
   int64_t q_rows;    // rows of the packed Qw tensor
   int64_t k_rows;    // rows of the packed K tensor

@@ -11,20 +11,21 @@
 //                            256-key tiles -> partial (m, z) per key split;
 //   merge  (lse_merge)       -lse2 = -(m + log2 z) over the splits (or minus
 //                            the caller's natural-log normaliser * log2 e),
-//                            written per (layer, KV head) in 128-row chunks
-//                            padded with -inf;
-//   pass 2 (score_colsum_tc) keys in TMEM lanes: each thread owns one key and
-//                            sums exp2(x*scale*log2e - lse2[row]) over all
-//                            rows of all layers (compensated), s = sum / L.
-//                            The chunk's normalisers arrive with its Q rows
-//                            (one bulk copy), padding rows contribute 0.
+//                            written per (layer, KV head) padded with -inf to
+//                            whole 256-row chunks;
+//   pass 2 (score_colsum_tc) CTA pairs, keys in TMEM lanes: each thread owns
+//                            one key and sums exp2(x*scale*log2e - lse2[row])
+//                            over all rows of all layers (compensated),
+//                            s = sum / L.  Each 256-row chunk's normalisers
+//                            arrive beside its Q rows (one bulk copy per
+//                            CTA), padding rows contribute 0.
 //
 // Warp roles in both passes (320 threads, one CTA per SM): warps 0-3 and 4-7
 // are two consumer warpgroups (one TMEM lane per thread), warp 8 issues TMA and
 // owns the tensor-memory allocation, one thread of warp 9 issues the MMAs (in
-// pass 1 only the even CTA of each pair issues them, as 2-SM MMAs: M = 256
-// rows, N = 256 keys, 128 cycles each, so the issuing thread's barrier waits
-// and commits hide behind the tensor pipe).
+// both passes only the even CTA of each pair issues them, as 2-SM MMAs of
+// M = N = 256, 128 cycles each, so the issuing thread's barrier waits and
+// commits hide behind the tensor pipe).
 // Each consumer thread takes a whole tile (up to 128 accumulators) per step,
 // so its exps and sums form many independent chains.  Every wait is bounded: on a
 // timeout the CTA stops issuing, waits for its own copies and MMAs, frees its
@@ -49,8 +50,6 @@ constexpr int kProducerWarp = 8, kMmaWarp = 9;
 constexpr uint32_t kTile = 128;                 // keys per tile, rows per block / chunk
 constexpr uint32_t kKBlockBytes = kTile * 128;  // 128 rows x 64 bf16
 constexpr uint32_t kTileBytes = 2 * kKBlockBytes;
-constexpr int kStages1 = 3;                     // K ring of pass 1
-constexpr int kQStages = 4;                     // Q ring of pass 2
 constexpr uint32_t kTmemCols = 512;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -341,61 +340,84 @@ __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __res
 }
 
 // ---------------------------------------------------------------------------
-// pass 2
+// pass 2 on CTA pairs
+//
+// A pair owns a tile of 256 keys (128 per CTA, keys in TMEM lanes) and walks
+// all layers: per layer its K rows (each CTA its own 128 keys, double
+// buffered), then the layer's window rows in chunks of 256 (each CTA loads
+// 128 rows of the chunk).  One 2-SM MMA chain (M = 256 keys, N = 256 rows,
+// K = 128) leaves each key's 256 logits in its own CTA's tensor memory.
+// Every CTA also loads the chunk's 256 row normalisers into its own shared
+// memory (rows past the row set carry -inf and add 0).  Warpgroup wg takes
+// the chunks q with q % 2 == wg (TMEM slot wg), all 256 columns in two
+// halves.
+
+constexpr uint32_t kChunkRows = 256;            // window rows per pass-2 chunk (both CTAs)
+constexpr int kQStagesPair = 4;                 // Q ring of pass 2 (per CTA: 32 KB + 1 KB a stage)
 
 struct P2Smem {
-  uint8_t k[2][2][kKBlockBytes];          // [stage = layer & 1][K-block]
-  uint8_t q[kQStages][2][kKBlockBytes];   // [stage][K-block]
-  float nlse[kQStages][kTile];            // minus lse2 of the stage's rows (-inf = padding)
-  float red[2][kTile];                    // [warpgroup][key]
-  uint64_t k_full[2], k_empty[2];
-  uint64_t q_full[kQStages], q_empty[kQStages];
-  uint64_t tm_full[kQStages], tm_empty[kQStages];
+  uint8_t k[2][2][kKBlockBytes];              // this CTA's 128 keys of layer l [l & 1][K-block]
+  uint8_t q[kQStagesPair][2][kKBlockBytes];   // this CTA's 128 rows of the chunk [stage][K-block]
+  float nlse[kQStagesPair][kChunkRows];       // minus lse2 of all 256 rows of the chunk
+  float red[2][kTile];                        // [warpgroup][key]
+  uint64_t k_full[2];                         // even CTA: both CTAs' keys of the layer landed
+  uint64_t k_empty[2];                        // both: the layer's MMAs are done
+  uint64_t q_full[kQStagesPair];              // even CTA: both CTAs' rows of the chunk landed
+  uint64_t nl_full[kQStagesPair];             // both: this CTA's copy of the normalisers landed
+  uint64_t q_empty[kQStagesPair];             // both: MMAs done and this CTA's warpgroup read the normalisers
+  uint64_t tm_full[2];                        // both: the slot's logits are ready
+  uint64_t tm_empty[2];                       // even CTA: the slot's 8 consumer warps copied it out
   uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
 };
 
-
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                        Shape sh, Tables tb, const float* __restrict__ nlse, float* __restrict__ scores) {
   extern __shared__ uint8_t smem_raw[];
   P2Smem& sm = *reinterpret_cast<P2Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int unit = (int)(blockIdx.x >> 1);
 
-  const int r = upper_index(tb.unit0_tc2, sh.n_req, (int32_t)blockIdx.x);
+  const int r = upper_index(tb.unit0_tc2, sh.n_req, (int32_t)unit);
   const Req rq = tb.req[r];
-  const int u = blockIdx.x - tb.unit0_tc2[r];
+  const int u = unit - tb.unit0_tc2[r];
   const int g = u / rq.tiles, kt = u % rq.tiles;
-  const int rows = sh.G * rq.W;
-  const int C = rq.C;
+  const int C = rq.C;                          // 128-row chunks per layer (even)
+  const int C2 = C >> 1;                       // 256-row chunks per layer
   const int L = sh.L;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
-    for (int i = 0; i < kQStages; ++i) {
-      mbar_init(&sm.q_full[i], 1);
-      mbar_init(&sm.q_empty[i], 1 + 4);   // MMA commit + one arrival per consumer warp
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.k_full[i], 1);
+      mbar_init(&sm.k_empty[i], 1);
       mbar_init(&sm.tm_full[i], 1);
-      mbar_init(&sm.tm_empty[i], kTile);
+      mbar_init(&sm.tm_empty[i], 8);
+    }
+    for (int i = 0; i < kQStagesPair; ++i) {
+      mbar_init(&sm.q_full[i], 1);
+      mbar_init(&sm.nl_full[i], 1);
+      mbar_init(&sm.q_empty[i], 1 + 4);   // MMA commit + the stage's 4 consumer warps of this CTA
     }
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (warp == kProducerWarp) {
-    tmem_alloc(&sm.tmem_base, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, kTmemCols);
+    tmem_relinquish_pair();
   }
+  __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
   if (warp == kProducerWarp && lane == 0) {
-    // ---- TMA producer: K tile of layer l, then the C row chunks of layer l
+    // ---- TMA producer (both CTAs): K half of layer l, then the layer's row chunks
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
     int k_issued = 0, q_issued = 0;
@@ -403,112 +425,127 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     for (int l = 0; ok && l < L; ++l) {
       const int ks = l & 1;
       if (!mbar_wait(&sm.k_empty[ks], ((l >> 1) & 1) ^ 1, abort)) break;
-      mbar_arrive_expect_tx(&sm.k_full[ks], kTileBytes);
-      const int ky = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + kt * (int)kTile;
-      tma_load_2d(sm.k[ks][0], &tmK, 0, ky, &sm.k_full[ks]);
-      tma_load_2d(sm.k[ks][1], &tmK, 64, ky, &sm.k_full[ks]);
+      if (rank == 0) mbar_arrive_expect_tx(&sm.k_full[ks], 2 * kTileBytes);
+      const uint32_t k_full0 = map_to_rank(smem_u32(&sm.k_full[ks]), 0);
+      const int ky = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + kt * (int)kPairKeys +
+                     (int)rank * (int)kTile;
+      tma_load_2d_pair(sm.k[ks][0], &tmK, 0, ky, k_full0);
+      tma_load_2d_pair(sm.k[ks][1], &tmK, 64, ky, k_full0);
       ++k_issued;
-      const int qy0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W);
-      for (int c = 0; c < C; ++c) {
-        const int q = l * C + c, qs = q % kQStages;
-        if (!mbar_wait(&sm.q_empty[qs], ((q / kQStages) & 1) ^ 1, abort)) { ok = false; break; }
-        mbar_arrive_expect_tx(&sm.q_full[qs], kTileBytes + kTile * 4);
-        tma_load_2d(sm.q[qs][0], &tmQ, 0, qy0 + c * (int)kTile, &sm.q_full[qs]);
-        tma_load_2d(sm.q[qs][1], &tmQ, 64, qy0 + c * (int)kTile, &sm.q_full[qs]);
-        bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C + c) * kTile,
-                  kTile * 4, &sm.q_full[qs]);
+      const int qy0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + (int)rank * (int)kTile;
+      for (int c = 0; c < C2; ++c) {
+        const int q = l * C2 + c, qs = q % kQStagesPair;
+        if (!mbar_wait(&sm.q_empty[qs], ((q / kQStagesPair) & 1) ^ 1, abort)) { ok = false; break; }
+        if (rank == 0) mbar_arrive_expect_tx(&sm.q_full[qs], 2 * kTileBytes);
+        const uint32_t q_full0 = map_to_rank(smem_u32(&sm.q_full[qs]), 0);
+        tma_load_2d_pair(sm.q[qs][0], &tmQ, 0, qy0 + c * (int)kChunkRows, q_full0);
+        tma_load_2d_pair(sm.q[qs][1], &tmQ, 64, qy0 + c * (int)kChunkRows, q_full0);
+        mbar_arrive_expect_tx(&sm.nl_full[qs], kChunkRows * 4);
+        bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C2 + c) * kChunkRows,
+                  kChunkRows * 4, &sm.nl_full[qs]);
         ++q_issued;
       }
     }
-    for (int i = max(0, k_issued - 2); i < k_issued; ++i) drain_wait(&sm.k_full[i & 1], (i >> 1) & 1);
-    for (int i = max(0, q_issued - kQStages); i < q_issued; ++i)
-      drain_wait(&sm.q_full[i % kQStages], (i / kQStages) & 1);
-  } else if (warp == kMmaWarp && lane == 0) {
-    // ---- MMA issuer: D[key][row] = K_tile . Q_chunk^T
+    // every copy this CTA started has landed before the pair may leave: the
+    // normalisers on this CTA's barriers, the tiles on the even CTA's
+    for (int i = max(0, q_issued - kQStagesPair); i < q_issued; ++i)
+      drain_wait(&sm.nl_full[i % kQStagesPair], (i / kQStagesPair) & 1);
+    if (rank == 0) {
+      for (int i = max(0, k_issued - 2); i < k_issued; ++i) drain_wait(&sm.k_full[i & 1], (i >> 1) & 1);
+      for (int i = max(0, q_issued - kQStagesPair); i < q_issued; ++i)
+        drain_wait(&sm.q_full[i % kQStagesPair], (i / kQStagesPair) & 1);
+    }
+  } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
+    // ---- MMA issuer (even CTA): D[key][row] = K_tile . Q_chunk^T, 256 x 256
+    const uint32_t idesc = idesc_bf16_f32(2 * kTile, kChunkRows);
     bool ok = true;
     for (int l = 0; ok && l < L; ++l) {
       const int ks = l & 1;
       if (!mbar_wait(&sm.k_full[ks], (l >> 1) & 1, abort)) break;
-      for (int c = 0; c < C; ++c) {
-        const int q = l * C + c, qs = q % kQStages;
-        const uint32_t use = (uint32_t)(q / kQStages);
-        if (!mbar_wait(&sm.q_full[qs], use & 1, abort)) { ok = false; break; }
-        if (!mbar_wait(&sm.tm_empty[qs], (use & 1) ^ 1, abort)) { ok = false; break; }
+      for (int c = 0; c < C2; ++c) {
+        const int q = l * C2 + c, qs = q % kQStagesPair, slot = q & 1;
+        if (!mbar_wait(&sm.q_full[qs], (q / kQStagesPair) & 1, abort)) { ok = false; break; }
+        if (!mbar_wait(&sm.tm_empty[slot], ((q >> 1) & 1) ^ 1, abort)) { ok = false; break; }
         tc_fence_after();
-        // always a full 128-row chunk: rows past the row set carry a -inf normaliser
-        const uint32_t idesc = idesc_bf16_f32(kTile, kTile);
-        const uint32_t d = tbase + (uint32_t)qs * kTile;
+        const uint32_t d = tbase + (uint32_t)slot * kChunkRows;
 #pragma unroll
         for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            mma_bf16(d, desc_sw128(smem_u32(sm.k[ks][kb]) + k * 32),
-                     desc_sw128(smem_u32(sm.q[qs][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
-        mma_commit(&sm.tm_full[qs]);
-        mma_commit(&sm.q_empty[qs]);
+            mma_bf16_pair(d, desc_sw128(smem_u32(sm.k[ks][kb]) + k * 32),
+                          desc_sw128(smem_u32(sm.q[qs][kb]) + k * 32), idesc, (kb | k) ? 1u : 0u);
+        mma_commit_pair(&sm.tm_full[slot], 3);
+        mma_commit_pair(&sm.q_empty[qs], 3);
       }
-      if (ok) mma_commit(&sm.k_empty[ks]);
+      if (ok) mma_commit_pair(&sm.k_empty[ks], 3);
     }
-    mma_commit(&sm.mma_done);
+    mma_commit_pair(&sm.mma_done, 1);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
-    // ---- column sums: one thread per key (= TMEM lane); warpgroup wg takes
-    // the chunks q = l*C + c with q % 2 == wg
+    // ---- column sums: one thread per key (= TMEM lane)
     const int wg = warp >> 2;
     const int key = ((warp & 3) << 5) + lane;
     const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
+    const uint32_t tm_empty0 = lane == 0 ? map_to_rank(smem_u32(&sm.tm_empty[wg]), 0) : 0u;
     const float s2 = sh.scale_log2;
-    const int v = kt * (int)kTile + key;
+    const int v = kt * (int)kPairKeys + (int)rank * (int)kTile + key;
     const bool per_layer = sh.rank_mode == VC_RANK_PER_LAYER;
-    const int nq = L * C;
+    const int nq = L * C2;
     Kahan tot, lay;
     tot.init();
     lay.init();
     for (int q = 0; q < nq; ++q) {
-      const int l = q / C, c = q % C;
+      const int l = q / C2, c = q % C2;
       if ((q & 1) == wg) {
-        const int qs = q % kQStages;
-        const uint32_t use = (uint32_t)(q / kQStages);
+        const int qs = q % kQStagesPair;
         const bool go = __all_sync(0xffffffffu, *abort == 0);
-        if (go && warp_wait(&sm.tm_full[qs], use & 1, abort)) {
+        if (go && warp_wait(&sm.tm_full[wg], (q >> 1) & 1, abort) &&
+            warp_wait(&sm.nl_full[qs], (q / kQStagesPair) & 1, abort)) {
           tc_fence_after();
-          const uint32_t col0 = tbase + lane_off + (uint32_t)qs * kTile;
-          float x[8][16];
-          {
-            uint32_t v[8][16];
+#pragma unroll 1
+          for (int hf = 0; hf < 2; ++hf) {
+            const uint32_t col0 = tbase + lane_off + (uint32_t)wg * kChunkRows + (uint32_t)hf * kTile;
+            float x[8][16];
+            {
+              uint32_t vv[8][16];
 #pragma unroll
-            for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, v[p]);
-            tmem_wait_only();
+              for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, vv[p]);
+              tmem_wait_only();
+#pragma unroll
+              for (int p = 0; p < 8; ++p) {
+                reg_fence(vv[p]);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(vv[p][j]);
+              }
+            }
+            if (hf == 1) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive_cluster(tm_empty0);   // slot copied out
+            }
+            const float4* nl = reinterpret_cast<const float4*>(sm.nlse[qs] + hf * (int)kTile);
+            float ps[8];
 #pragma unroll
             for (int p = 0; p < 8; ++p) {
-              reg_fence(v[p]);
+              float2 nb[8];
 #pragma unroll
-              for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(v[p][j]);
+              for (int j = 0; j < 4; ++j) {
+                const float4 f = nl[p * 4 + j];
+                nb[2 * j] = make_float2(f.x, f.y);
+                nb[2 * j + 1] = make_float2(f.z, f.w);
+              }
+              ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
             }
+            lay.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
           }
-          tc_fence_before();
-          mbar_arrive(&sm.tm_empty[qs]);
-          const float4* nl = reinterpret_cast<const float4*>(sm.nlse[qs]);
-          float ps[8];
-#pragma unroll
-          for (int p = 0; p < 8; ++p) {
-            float2 nb[8];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float4 f = nl[p * 4 + j];
-              nb[2 * j] = make_float2(f.x, f.y);
-              nb[2 * j + 1] = make_float2(f.z, f.w);
-            }
-            ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
-          }
-          lay.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.q_empty[qs]);   // this warp is done with the stage's normalisers
       }
-      if (c == C - 1) {
+      if (c == C2 - 1) {
         if (per_layer) {
           sm.red[wg][key] = lay.s;
+          __syncwarp();
           named_sync(1, 2 * kTile);
           if (wg == 0 && v < rq.n)
             scores[rq.s_off + ((int64_t)l * sh.Hkv + g) * rq.n + v] = sm.red[0][key] + sm.red[1][key];
@@ -521,17 +558,18 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     }
     if (!per_layer) {
       sm.red[wg][key] = tot.s;
+      __syncwarp();
       named_sync(1, 2 * kTile);
       if (wg == 0 && v < rq.n)
         scores[rq.s_off + (int64_t)g * rq.n + v] = (sm.red[0][key] + sm.red[1][key]) / (float)L;
     }
   }
+  __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();                  // no CTA leaves while the pair's MMAs or copies may touch it
   if (warp == kProducerWarp) {
-    __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tbase, kTmemCols);
+    tmem_dealloc_pair(tbase, kTmemCols);
   }
   if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
 }
@@ -623,7 +661,7 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
   e = cudaFuncSetAttribute(score_colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   if (e != cudaSuccess) return e;
   ProfileScope ps("score_colsum_tc", st);
-  score_colsum_tc_kernel<<<tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, nlse_pad, scores);
+  score_colsum_tc_kernel<<<2 * tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, nlse_pad, scores);
   return cudaGetLastError();
 }
 

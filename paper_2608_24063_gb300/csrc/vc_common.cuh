@@ -23,9 +23,10 @@ struct Req {                 // one request of a batch
   int64_t lsep_off;          // float offset of its chunk-padded row normalisers [L][Hkv][C*128]
   int64_t vs_row0;           // first row of its compacted survivors' values (tensor-core fusion)
   int32_t n, W, Nq, h;
-  int32_t C;                 // 128-row chunks of one (layer, KV head) row set, ceil(G*W/128)
+  int32_t C;                 // 128-row chunks of one (layer, KV head) row set, padded to
+                             // whole 256-row chunks: 2*ceil(G*W/256)
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
-  int32_t tiles;             // 128-key tiles, ceil(n/128)
+  int32_t tiles;             // 256-key tiles, ceil(n/256)
   int32_t pad_;
 };
 

@@ -5,18 +5,14 @@
 //   kept key rows go to K_out (bit-exact), and the survivors' value rows --
 //   kept then dropped, each list in ascending position -- are compacted into a
 //   dense workspace slab Vs, so the fusion can stream them with TMA.
-// fuse_v_tc_kernel: one CTA per (request, layer, KV head, 256 kept rows):
+// fuse_v_tc_kernel: one CTA pair per (request, layer, KV head, 256 kept rows):
 //   O = softmax_row(V_k V_d^T / tau) V_d online over tiles of 128 dropped rows,
-//   V_out = mu V_k + (1 - mu) O.
-//   V_k and V_d tiles arrive by TMA (128-byte swizzle); S = V_k V_d^T and
-//   O += P V_d run on tcgen05.mma with fp32 accumulators in tensor memory (V_d
-//   read K-major for the first product, MN-major for the second), P goes
-//   through shared memory in bf16.  The softmax keeps a per-row reference
-//   maximum and rescales O in tensor memory only when a tile's maximum exceeds
-//   it by more than 2^8.
-//   Warp roles (320 threads, one CTA per SM): warps 0-3 and 4-7 own one kept
-//   row each (= TMEM lane), warp 8 issues TMA and owns the tensor memory, one
-//   thread of warp 9 issues the MMAs.  Every wait is bounded (tc_common.cuh).
+//   V_out = mu V_k + (1 - mu) O, on 2-SM tcgen05.mma with fp32 accumulators in
+//   tensor memory; the numerators P go from the softmax warps to the second
+//   product through tensor memory.  Warp roles (320 threads, two CTAs per SM):
+//   warps 0-7 softmax and epilogue, warp 8 TMA and the tensor-memory
+//   allocation, one thread of warp 9 (even CTA) the MMAs.  Every wait is
+//   bounded (tc_common.cuh).
 #include <cudaTypedefs.h>
 
 #include <mutex>
@@ -64,25 +60,52 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// fusion
+// fusion on CTA pairs
+//
+// A pair owns 256 kept rows of one (request, layer, KV head) (CTA r: rows
+// r*128 ... r*128+127, one per TMEM lane) and streams the dropped rows in
+// tiles of 128.  Per tile j the even CTA issues
+//   S = V_k V_d(j)^T   2-SM MMA, M = 256, N = 128 dropped rows (CTA r stages
+//                      dropped rows r*64 ... r*64+63, K-major),
+//   O += P(j) V_d(j)   2-SM MMA, M = 256, N = 128 value columns (CTA r stages
+//                      columns r*64 ... r*64+63 of all 128 dropped rows,
+//                      MN-major), A = P read from tensor memory,
+// in the order S(0), [P(0) ready] O(0), S(1), [P(1) ready] O(1), ...  P(j) is
+// written in bf16 over the first half of each softmax warp's own S columns,
+// so S(j+1) (issued after O(j)) may reuse them.  Two pairs run per TPC, so
+// one pair's softmax and prologue overlap the other's MMAs.
+//
+// Tensor memory per CTA (256 columns): O in [0, 128), S / P in [128, 256).
+// Softmax: warps w and w+4 share the TMEM lanes of warp w % 4; warp w takes
+// S columns 0-63 (dropped rows 0-63 of the tile), warp w+4 columns 64-127.
+// They agree on the row's reference maximum through shared memory each
+// tile; the maximum is raised (and O rescaled in tensor memory) only when a
+// tile exceeds it by more than 2^8.
 
 constexpr int kThreads = 320;
 constexpr int kProducerWarp = 8, kMmaWarp = 9;
 constexpr uint32_t kTile = 128;
-constexpr uint32_t kKB = kTile * 128;            // one K-block: 128 rows x 128 bytes
-constexpr uint32_t kTileBytes = 2 * kKB;
-constexpr int kVdStages = 3;
-constexpr uint32_t kTmemCols = 512;              // O_0, O_1, S_0, S_1: 128 columns each
+constexpr uint32_t kKB = kTile * 128;            // 128 rows x 128 bytes
+constexpr uint32_t kHalfKB = 64 * 128;           // 64 rows x 128 bytes
+constexpr int kVdStages = 2;
+constexpr uint32_t kTmemCols = 256;              // O: [0,128), S/P: [128,256)
+constexpr uint32_t kSCol = 128;
 constexpr float kRescaleLog2 = 8.f;
 
 struct FSmem {
-  uint8_t vk[2][2][kKB];              // [half][K-block] kept rows: A operand of S = V_k V_d^T
-  uint8_t vd[kVdStages][2][kKB];      // dropped rows: B operand of both products
-  uint8_t p[2][2][kKB];               // [half][K-block] numerators (bf16): A of O += P V_d
-  uint64_t vk_full;
-  uint64_t vd_full[kVdStages], vd_empty[kVdStages];
-  uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2];
-  uint64_t o_full, mma_done;
+  uint8_t vk[2][kKB];                 // this CTA's 128 kept rows [K-block]: A of S = V_k V_d^T
+  uint8_t vds[kVdStages][2][kHalfKB]; // this CTA's 64 dropped rows [stage][K-block]: B of S
+  uint8_t vdo[kVdStages][kKB];        // all 128 dropped rows, this CTA's 64 columns: B of O += P V_d
+  float xmax[2][4][2][32];            // [tile & 1][lane quadrant][column half][lane]: tile maxima
+  float lsum[2][4][32];               // [column half][lane quadrant][lane]: partial row sums
+  uint64_t vk_own;                    // this CTA's kept rows landed
+  uint64_t vk_pair;                   // even CTA: both CTAs' kept rows landed (2 arrivals)
+  uint64_t vd_full[kVdStages];        // even CTA: both CTAs' dropped tiles landed
+  uint64_t vd_empty[kVdStages];       // both: the MMAs reading the stage are done
+  uint64_t s_full;                    // both: S(j) is in tensor memory (and O(j-1) done)
+  uint64_t p_full;                    // even CTA: all 16 softmax warps wrote P(j)
+  uint64_t o_full;                    // both: the last O product is done
+  uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
 };
@@ -102,10 +125,10 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, ok);
 }
 
-// Byte offset of 16-byte chunk c (0..15) of row r in a swizzled 128-row tile pair
-// (the 128-byte swizzle TMA writes and the MMA descriptors expect).
+// Byte offset of 16-byte chunk c (0..7) of row r in a 128-byte-swizzled
+// K-block (the layout TMA writes and the MMA descriptors expect).
 __device__ __forceinline__ uint32_t swz(int r, int c) {
-  return (uint32_t)((c >> 3) * kKB + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+  return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
@@ -113,23 +136,24 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmVs, Shape sh, Tables tb, float mu, float c2,
-                 __nv_bfloat16* __restrict__ V_out) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 2)
+fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_constant__ CUtensorMap tmRows64,
+                 Shape sh, Tables tb, float mu, float c2, __nv_bfloat16* __restrict__ V_out) {
   extern __shared__ uint8_t smem_raw[];
   FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int unit = (int)(blockIdx.x >> 1);
 
-  const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)blockIdx.x);
-  const int r = rl / sh.L, l = rl % sh.L;
+  const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
+  const int r = rl / sh.L;
   const Req rq = tb.req[r];
   const Layer ly = tb.layer[rl];
   const int ktiles = (ly.B + 2 * (int)kTile - 1) / (2 * (int)kTile);
-  const int u = blockIdx.x - tb.unit0_fuse_tc[rl];
+  const int u = unit - tb.unit0_fuse_tc[rl];
   const int g = u / ktiles;
-  const int r0 = (u % ktiles) * 2 * (int)kTile;
-  const int rows = min(2 * (int)kTile, ly.B - r0);        // kept rows of this CTA
-  const int nhalf = rows > (int)kTile ? 2 : 1;            // halves with kept rows
+  const int r0 = (u % ktiles) * 2 * (int)kTile + (int)rank * (int)kTile;   // this CTA's first kept row
+  const int rows = max(0, min((int)kTile, ly.B - r0));                    // kept rows of this CTA
   const int D = ly.D;
   const int nt = (D + (int)kTile - 1) / (int)kTile;
   // rows of this (layer, KV head) in Vs: B kept, then D dropped
@@ -137,142 +161,167 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmVs, Shape sh, Tables tb, 
   const int64_t orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
 
   if (threadIdx.x == 0) {
-    mbar_init(&sm.vk_full, 1);
+    mbar_init(&sm.vk_own, 1);
+    mbar_init(&sm.vk_pair, 2);
     for (int i = 0; i < kVdStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.s_full[i], 1);
-      mbar_init(&sm.s_empty[i], kTile);
-      mbar_init(&sm.p_full[i], kTile);
-      mbar_init(&sm.p_empty[i], 1);
-    }
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.p_full, 16);
     mbar_init(&sm.o_full, 1);
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (warp == kProducerWarp) {
-    tmem_alloc(&sm.tmem_base, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&sm.tmem_base, kTmemCols);
+    tmem_relinquish_pair();
   }
+  __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
-  if (warp == kProducerWarp) {
-    if (lane == 0) {
-      // ---- TMA producer: the kept rows once, then a ring of dropped-row tiles
-      prefetch_tmap(&tmVs);
-      mbar_arrive_expect_tx(&sm.vk_full, nhalf * kTileBytes);
-      for (int h = 0; h < nhalf; ++h)
-        for (int kb = 0; kb < 2; ++kb)
-          tma_load_2d(sm.vk[h][kb], &tmVs, kb * 64, vs0 + r0 + h * (int)kTile, &sm.vk_full);
-      int issued = 0;
-      for (int j = 0; j < nt; ++j) {
-        const int st = j % kVdStages;
-        if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
-        mbar_arrive_expect_tx(&sm.vd_full[st], kTileBytes);
-        const int y = vs0 + ly.B + j * (int)kTile;
-        tma_load_2d(sm.vd[st][0], &tmVs, 0, y, &sm.vd_full[st]);
-        tma_load_2d(sm.vd[st][1], &tmVs, 64, y, &sm.vd_full[st]);
-        ++issued;
+  if (warp == kProducerWarp && lane == 0) {
+    // ---- TMA producer (both CTAs)
+    prefetch_tmap(&tmRows128);
+    prefetch_tmap(&tmRows64);
+    mbar_arrive_expect_tx(&sm.vk_own, 2 * kKB);
+    for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.vk[kb], &tmRows128, kb * 64, vs0 + r0, &sm.vk_own);
+    int issued = 0;
+    for (int j = 0; j < nt; ++j) {
+      if (j == kVdStages) {
+        // the ring is full: own kept rows landed -> tell the even CTA, whose
+        // MMAs read them (and must run before any stage frees up)
+        if (!mbar_wait(&sm.vk_own, 0, abort)) break;
+        mbar_arrive_cluster(map_to_rank(smem_u32(&sm.vk_pair), 0));
       }
-      drain_wait(&sm.vk_full, 0);
+      const int st = j % kVdStages;
+      if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
+      if (rank == 0) mbar_arrive_expect_tx(&sm.vd_full[st], 2 * (2 * kHalfKB + kKB));
+      const uint32_t full0 = map_to_rank(smem_u32(&sm.vd_full[st]), 0);
+      const int y = vs0 + ly.B + j * (int)kTile;
+      tma_load_2d_pair(sm.vds[st][0], &tmRows64, 0, y + (int)rank * 64, full0);
+      tma_load_2d_pair(sm.vds[st][1], &tmRows64, 64, y + (int)rank * 64, full0);
+      tma_load_2d_pair(sm.vdo[st], &tmRows128, (int)rank * 64, y, full0);
+      ++issued;
+    }
+    if (nt <= kVdStages && mbar_wait(&sm.vk_own, 0, abort))
+      mbar_arrive_cluster(map_to_rank(smem_u32(&sm.vk_pair), 0));
+    if (rank == 0)
       for (int i = max(0, issued - kVdStages); i < issued; ++i)
         drain_wait(&sm.vd_full[i % kVdStages], (i / kVdStages) & 1);
-    }
-  } else if (warp == kMmaWarp) {
-    if (lane == 0) {
-      // ---- MMA issuer.  Per drop tile j: S_h = V_k,h V_d(j)^T for both halves,
-      // then O_h += P_h(j-1) V_d(j-1) for both halves.
-      const uint32_t id_s = idesc_bf16_f32(kTile, kTile);
-      const uint32_t id_o = idesc_bf16_f32_bmn(kTile, kTile);
-      bool ok = mbar_wait(&sm.vk_full, 0, abort);
-      for (int j = 0; ok && j <= nt; ++j) {
-        if (j < nt) {
-          const int st = j % kVdStages;
-          if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
-          for (int h = 0; h < nhalf && ok; ++h) {
-            if (!mbar_wait(&sm.s_empty[h], (j & 1) ^ 1, abort)) { ok = false; break; }
-            tc_fence_after();
-            const uint32_t d = tbase + (uint32_t)(2 + h) * kTile;
+  } else if (warp == kMmaWarp && lane == 0 && rank == 0 && nt > 0) {
+    // ---- MMA issuer (even CTA)
+    const uint32_t id_s = idesc_bf16_f32(2 * kTile, kTile);
+    const uint32_t id_o = idesc_bf16_f32_bmn(2 * kTile, kTile);
+    const uint32_t s_tm = tbase + kSCol;
+    bool ok = mbar_wait(&sm.vk_pair, 0, abort);
+    int jo = 0;                                   // next O product to issue
+    for (int j = 0; ok && j <= nt; ++j) {
+      if (j >= 1) {
+        // O += P(j-1) V_d(j-1), once the softmax has written P(j-1)
+        if (!mbar_wait(&sm.p_full, (j - 1) & 1, abort)) break;
+        tc_fence_after();
+        const int st = (j - 1) % kVdStages;
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16(d, desc_sw128(smem_u32(sm.vk[h][kk >> 2]) + (kk & 3) * 32),
-                       desc_sw128(smem_u32(sm.vd[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
-            mma_commit(&sm.s_full[h]);
-          }
-          if (!ok) break;
-        }
-        if (j >= 1) {
-          const int jp = j - 1, st = jp % kVdStages;
-          for (int h = 0; h < nhalf && ok; ++h) {
-            if (!mbar_wait(&sm.p_full[h], jp & 1, abort)) { ok = false; break; }
-            tc_fence_after();
-            const uint32_t d = tbase + (uint32_t)h * kTile;
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16(d, desc_sw128(smem_u32(sm.p[h][kk >> 2]) + (kk & 3) * 32),
-                       desc_sw128_mn(smem_u32(sm.vd[st][0]) + kk * 2048, kKB), id_o,
-                       (jp > 0 || kk > 0) ? 1u : 0u);
-            mma_commit(&sm.p_empty[h]);
-          }
-          if (ok) mma_commit(&sm.vd_empty[st]);
-        }
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_pair_ta(tbase, s_tm + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
+                           desc_sw128_mn(smem_u32(sm.vdo[st]) + kk * 2048, kKB), id_o,
+                           (j > 1 || kk > 0) ? 1u : 0u);
+        mma_commit_pair(&sm.vd_empty[st], 3);
+        jo = j;
       }
-      mma_commit(&sm.o_full);
-      mma_commit(&sm.mma_done);
-      drain_wait(&sm.mma_done, 0);
+      if (j < nt) {
+        // S(j) = V_k V_d(j)^T (after O(j-1) in the pipe, so P(j-1) has been read)
+        const int st = j % kVdStages;
+        if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16_pair(s_tm, desc_sw128(smem_u32(sm.vk[kk >> 2]) + (kk & 3) * 32),
+                        desc_sw128(smem_u32(sm.vds[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
+        mma_commit_pair(&sm.s_full, 3);
+      }
     }
-  } else {
-    // ---- softmax over the drop set and epilogue: one thread per kept row
-    const int h = warp >> 2;                              // half of the kept tile
-    const int row = ((warp & 3) << 5) + lane;             // row within the half = TMEM lane
-    const uint32_t lane_off = (uint32_t)((warp & 3) << 5) << 16;
-    const uint32_t o_col = tbase + lane_off + (uint32_t)h * kTile;
-    const uint32_t s_col = tbase + lane_off + (uint32_t)(2 + h) * kTile;
-    const bool active = h < nhalf;
+    if (jo == nt) mma_commit_pair(&sm.o_full, 3);
+    mma_commit_pair(&sm.mma_done, 1);
+    drain_wait(&sm.mma_done, 0);
+  } else if (warp < 8) {
+    // ---- softmax over the drop set and epilogue: one kept row per TMEM lane
+    const int q4 = warp & 3;                          // lane quadrant
+    const int hf = warp >> 2;                         // column half
+    const int row = (q4 << 5) + lane;                 // row within this CTA's 128
+    const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
+    const uint32_t o_col = tbase + lane_off + (uint32_t)hf * 64;
+    const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)hf * 64;
+    const uint32_t p_full0 = lane == 0 ? map_to_rank(smem_u32(&sm.p_full), 0) : 0u;
     float m = -INFINITY, lsum = 0.f;
     bool ok = true;
-    for (int j = 0; active && j < nt; ++j) {
-      if (!warp_wait(&sm.s_full[h], j & 1, abort)) { ok = false; break; }
+    for (int j = 0; j < nt; ++j) {
+      if (!warp_wait(&sm.s_full, j & 1, abort)) { ok = false; break; }
       tc_fence_after();
-      uint32_t xs[8][16];                                 // S row of this thread (fp32 bits)
+      float x[4][16];
+      {
+        uint32_t v[4][16];
 #pragma unroll
-      for (int p = 0; p < 8; ++p) tmem_ld16(s_col + p * 16, xs[p]);
-      tmem_wait_only();
+        for (int p = 0; p < 4; ++p) tmem_ld16(s_col + p * 16, v[p]);
+        tmem_wait_only();
 #pragma unroll
-      for (int p = 0; p < 8; ++p) reg_fence(xs[p]);
-      tc_fence_before();
-      mbar_arrive(&sm.s_empty[h]);                        // S copied out: the next product may start
-      const int valid = min((int)kTile, D - j * (int)kTile);
-      if (valid < (int)kTile) {                           // last tile: drop columns past D
+        for (int p = 0; p < 4; ++p) {
+          reg_fence(v[p]);
 #pragma unroll
-        for (int p = 0; p < 8; ++p)
+          for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
+        }
+      }
+      const int valid = min(64, D - j * (int)kTile - hf * 64);
+      if (valid < 64) {                               // last tile: columns past D
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
 #pragma unroll
           for (int q = 0; q < 16; ++q)
-            if (p * 16 + q >= valid) xs[p][q] = 0xff800000u;   // -inf
+            if (p * 16 + q >= valid) x[p][q] = -INFINITY;
       }
-      float pm[8];
+      float a0 = fmaxf(x[0][0], x[0][1]), a1 = fmaxf(x[1][0], x[1][1]);
+      float a2 = fmaxf(x[2][0], x[2][1]), a3 = fmaxf(x[3][0], x[3][1]);
 #pragma unroll
-      for (int p = 0; p < 8; ++p) {
-        float a = fmaxf(__uint_as_float(xs[p][0]), __uint_as_float(xs[p][1]));
-#pragma unroll
-        for (int q = 2; q < 16; q += 2) a = fmax3(a, __uint_as_float(xs[p][q]), __uint_as_float(xs[p][q + 1]));
-        pm[p] = a;
+      for (int q = 2; q < 16; q += 2) {
+        a0 = fmax3(a0, x[0][q], x[0][q + 1]);
+        a1 = fmax3(a1, x[1][q], x[1][q + 1]);
+        a2 = fmax3(a2, x[2][q], x[2][q + 1]);
+        a3 = fmax3(a3, x[3][q], x[3][q + 1]);
       }
-      const float tm = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7])) * c2;
-      // raise the reference maximum when this tile exceeds it by more than 2^8
+      // this row's tile maximum over both column halves
+      sm.xmax[j & 1][q4][hf][lane] = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
+      named_sync(1 + q4, 64);
+      const float tm = fmaxf(sm.xmax[j & 1][q4][0][lane], sm.xmax[j & 1][q4][1][lane]) * c2;
       const bool raise = tm > m + kRescaleLog2;
       const float m_new = raise ? tm : m;
-      const float corr = raise ? ex2(m - m_new) : 1.f;     // 0 on the first tile
-      // the previous product must be done before P is rewritten (and before O is rescaled)
-      if (!warp_wait(&sm.p_empty[h], (j & 1) ^ 1, abort)) { ok = false; break; }
+      const float corr = raise ? ex2(m - m_new) : 1.f;   // 0 on the first tile
+      lsum *= corr;
+      m = m_new;
+      // P = exp2(S * c2 - m) in bf16 over the first 32 of this warp's S columns
+      const float2 sc = make_float2(c2, c2), nm = make_float2(-m, -m);
+      float2 ls = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int hp = 0; hp < 2; ++hp) {
+        uint32_t w[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          const int c = hp * 32 + 2 * q;
+          const float2 t = __ffma2_rn(make_float2(x[c >> 4][c & 15], x[c >> 4][(c & 15) + 1]), sc, nm);
+          const float2 e = make_float2(ex2(t.x), ex2(t.y));
+          ls = __fadd2_rn(ls, e);
+          w[q] = pack_bf16x2(e.x, e.y);
+        }
+        tmem_st16(s_col + hp * 16, w);
+      }
+      lsum += ls.x + ls.y;
       if (__any_sync(0xffffffffu, raise && j > 0)) {
-        tc_fence_after();
+        // rare: O(j-1) is complete (S(j) was issued after it) and O(j) waits
+        // for P(j); rescale this warp's 64 columns of O in tensor memory
 #pragma unroll 1
-        for (int p = 0; p < 8; ++p) {                    // rare: 16 columns at a time
+        for (int p = 0; p < 4; ++p) {
           uint32_t v[16];
           tmem_ld16(o_col + p * 16, v);
           tmem_wait(v);
@@ -280,90 +329,84 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmVs, Shape sh, Tables tb, 
           for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
           tmem_st16(o_col + p * 16, v);
         }
-        tmem_wait_st();
       }
-      lsum *= corr;
-      m = m_new;
-      // numerators in bf16 into the P tile (swizzled K-major A operand)
-      uint8_t* pt = &sm.p[h][0][0];
-      float2 ls = make_float2(0.f, 0.f);
-      const float2 sc = make_float2(c2, c2), nm = make_float2(-m, -m);
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        float e[8];
-#pragma unroll
-        for (int q = 0; q < 8; q += 2) {
-          const float2 t = __ffma2_rn(make_float2(__uint_as_float(xs[c >> 1][(c & 1) * 8 + q]),
-                                                  __uint_as_float(xs[c >> 1][(c & 1) * 8 + q + 1])), sc, nm);
-          e[q] = ex2(t.x);
-          e[q + 1] = ex2(t.y);
-          ls = __fadd2_rn(ls, make_float2(e[q], e[q + 1]));
-        }
-        uint4 w;
-        w.x = pack_bf16x2(e[0], e[1]);
-        w.y = pack_bf16x2(e[2], e[3]);
-        w.z = pack_bf16x2(e[4], e[5]);
-        w.w = pack_bf16x2(e[6], e[7]);
-        *reinterpret_cast<uint4*>(pt + swz(row, c)) = w;
-      }
-      lsum += ls.x + ls.y;
-      fence_proxy_async();
+      tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(&sm.p_full[h]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(p_full0);
     }
-    // epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped
-    const bool have_k = warp_wait(&sm.vk_full, 0, abort);
-    const bool have_o = active && have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
+    // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped
+    sm.lsum[hf][q4][lane] = lsum;
+    const bool have_k = warp_wait(&sm.vk_own, 0, abort);
+    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
+    __syncwarp();
+    named_sync(5, 256);
+    const float lt = sm.lsum[0][q4][lane] + sm.lsum[1][q4][lane];   // same order in both halves
     if (have_o) tc_fence_after();
-    const float w_o = have_o ? (1.f - mu) / lsum : 0.f;
+    const float w_o = have_o ? (1.f - mu) / lt : 0.f;
     const float w_k = have_o ? mu : 1.f;
-    const int grow = h * (int)kTile + row;                // row within the CTA's kept tile
+    // stage the 128 x 128 output tile in the (now idle) dropped-row buffers:
+    // row r at r * 256 bytes, 16-byte chunk c at slot c ^ (r & 15)
+    uint8_t* stage = &sm.vdo[0][0];
 #pragma unroll 1
-    for (int hh = 0; hh < 2; ++hh) {
-      float o[4][16];
+    for (int hh = 0; hh < 2; ++hh) {                  // 32 of this warp's 64 columns at a time
+      float o[2][16];
       if (have_o) {
-        uint32_t v[4][16];
+        uint32_t v[2][16];
 #pragma unroll
-        for (int p = 0; p < 4; ++p) tmem_ld16(o_col + hh * 64 + p * 16, v[p]);
+        for (int p = 0; p < 2; ++p) tmem_ld16(o_col + hh * 32 + p * 16, v[p]);
         tmem_wait_only();
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
+        for (int p = 0; p < 2; ++p) {
           reg_fence(v[p]);
 #pragma unroll
           for (int q = 0; q < 16; ++q) o[p][q] = __uint_as_float(v[p][q]);
         }
       } else {
 #pragma unroll
-        for (int p = 0; p < 4; ++p)
+        for (int p = 0; p < 2; ++p)
 #pragma unroll
           for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
       }
-      if (have_k && grow < rows) {
+      if (have_k) {
 #pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          const int c = hh * 8 + c8;
-          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[h][0][0] + swz(row, c));
+        for (int c4 = 0; c4 < 4; ++c4) {
+          const int c8 = hh * 4 + c4;                 // 16-byte chunk within the K-block
+          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[hf][0] + swz(row, c8));
           const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
           uint4 w;
           uint32_t* wp = &w.x;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float2 kf = __bfloat1622float2(k2[q]);
-            const float a = fmaf(w_k, kf.x, w_o * o[c8 >> 1][(c8 & 1) * 8 + 2 * q]);
-            const float b = fmaf(w_k, kf.y, w_o * o[c8 >> 1][(c8 & 1) * 8 + 2 * q + 1]);
+            const float a = fmaf(w_k, kf.x, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q]);
+            const float b = fmaf(w_k, kf.y, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q + 1]);
             wp[q] = pack_bf16x2(a, b);
           }
-          *reinterpret_cast<uint4*>(V_out + (orow + grow) * 128 + c * 8) = w;
+          const int c = hf * 8 + c8;
+          *reinterpret_cast<uint4*>(stage + row * 256 + ((c ^ (row & 15)) << 4)) = w;
         }
       }
     }
+    named_sync(5, 256);
+    // coalesced copy-out: 16 threads per 256-byte row
+    const int t = threadIdx.x;                        // 0..255
+    if (have_k) {
+#pragma unroll 4
+      for (int i = 0; i < 8; ++i) {
+        const int rr = i * 16 + (t >> 4), c = t & 15;
+        if (rr < rows)
+          *reinterpret_cast<uint4*>(V_out + (orow + rr) * 128 + c * 8) =
+              *reinterpret_cast<const uint4*>(stage + rr * 256 + ((c ^ (rr & 15)) << 4));
+      }
+    }
   }
+  __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();                  // no CTA leaves while the pair's MMAs or copies may touch it
   if (warp == kProducerWarp) {
-    __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tbase, kTmemCols);
+    tmem_dealloc_pair(tbase, kTmemCols);
   }
   if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
 }
@@ -382,12 +425,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows) {
+// [rows][128] bf16 tensor, boxes of box_rows rows x 64 elements, 128-byte swizzle.
+bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows, uint32_t box_rows) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
   if (!enc || rows == 0 || rows > 0x7fffffffull) return false;
   cuuint64_t dims[2] = {128, rows};
   cuuint64_t strides[1] = {256};
-  cuuint32_t box[2] = {64, kTile};
+  cuuint32_t box[2] = {64, box_rows};
   cuuint32_t es[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -412,15 +456,16 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  CUtensorMap mv;
-  if (!make_rows_map(&mv, Vs, (uint64_t)vs_rows)) return cudaErrorInvalidValue;
+  CUtensorMap m128, m64;
+  if (!make_rows_map(&m128, Vs, (uint64_t)vs_rows, kTile) || !make_rows_map(&m64, Vs, (uint64_t)vs_rows, 64))
+    return cudaErrorInvalidValue;
   const size_t smem = sizeof(FSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(fuse_v_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   ProfileScope ps("fuse_v_tc", st);
-  fuse_v_tc_kernel<<<units, kThreads, smem, st>>>(mv, sh, tb, mu, kLog2e / tau,
-                                                  static_cast<__nv_bfloat16*>(V_out));
+  fuse_v_tc_kernel<<<2 * units, kThreads, smem, st>>>(m128, m64, sh, tb, mu, kLog2e / tau,
+                                                      static_cast<__nv_bfloat16*>(V_out));
   return cudaGetLastError();
 }
 

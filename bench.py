@@ -103,21 +103,21 @@ KERNEL_WORK = {
 
 
 def traffic_for(kernel):
-    """dram bytes per launch from a committed ncu summary, if the kernel source is unchanged."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    """dram bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.md")
     if not os.path.exists(path):
         return None
-    with open(path) as f:
-        tab = json.load(f)
-    ent = tab.get(kernel)
-    if not ent:
-        return None
-    src = os.path.join(ROOT, ent["source"])
-    if not os.path.exists(src):
-        return None
-    with open(src, "rb") as f:
-        digest = hashlib.sha256(f.read()).hexdigest()[:16]
-    return ent["dram_bytes_per_launch"] if digest == ent["source_sha256_16"] else None
+    for line in open(path):
+        cells = [c.strip() for c in line.strip().strip("|").split("|")]
+        if len(cells) != 4 or cells[0] != kernel:
+            continue
+        src = os.path.join(ROOT, cells[1])
+        if not os.path.exists(src):
+            return None
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()[:16]
+        return int(cells[3]) if digest == cells[2] else None
+    return None
 
 
 # ---------------------------------------------------------------------------

@@ -227,6 +227,28 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
+def rank_workload(wl, rank):
+    """The workload one rank compresses under weak scaling: the same shapes and
+    request mix, its own requests (the seed offset by the rank)."""
+    import dataclasses
+    return wl if rank == 0 else dataclasses.replace(wl, seed=wl.seed + 7919 * rank)
+
+
+def max_over_ranks(x, world, dist, device):
+    """Max of a host float over all ranks (the timed region is the slowest rank's)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(units_per_rank, world, ms_per_step):
+    """Whole-job throughput: units of all ranks / the slowest rank's step time."""
+    return world * units_per_rank / (ms_per_step * 1e-3)
+
+
 def workload_config(wl):
     r = wl.requests[0]
     in_bytes = sum(wl.L * (wl.Hq * q.W + 2 * wl.Hkv * q.n) * wl.d * (2 if wl.dtype == "bf16" else 4)
@@ -262,7 +284,7 @@ def main():
     st = torch.cuda.current_stream()
 
     # inputs: generated on the device, resident in HBM before timing
-    qs, ks, vs = synth.generate(wl, dev)
+    qs, ks, vs = synth.generate(rank_workload(wl, rank), dev)
     Q = torch.cat([q.flatten() for q in qs]) if len(qs) > 1 else qs[0]
     K = torch.cat([k.flatten() for k in ks]) if len(ks) > 1 else ks[0]
     V = torch.cat([v.flatten() for v in vs]) if len(vs) > 1 else vs[0]
@@ -301,17 +323,13 @@ def main():
     kern = vc.viscache_profile_read()
     vc.viscache_profile_enable(False)
     clk = clocks.stop()
-    ms = t0.elapsed_time(t1)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(t0.elapsed_time(t1), world, dist, dev)
     ms_step = ms / args.steps
     assert vc.prunekv_get_status(ws) == vc.VC_OK
 
     plans = plans_for(wl, vc)
     work = algorithmic(wl, plans)
-    value = world * work["tokens_layers"] / (ms_step * 1e-3)
+    value = job_value(work["tokens_layers"], world, ms_step)
     pk = peaks()
 
     # dominant kernel
@@ -373,12 +391,8 @@ def main():
             e2e_step()
         b.record(st)
         torch.cuda.synchronize()
-        ems = a.elapsed_time(b) / e_steps
-        if world > 1:
-            tt = torch.tensor([ems], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ems = float(tt.item())
-        e2e = {"value": world * work["tokens_layers"] / (ems * 1e-3), "unit": UNIT,
+        ems = max_over_ranks(a.elapsed_time(b) / e_steps, world, dist, dev)
+        e2e = {"value": job_value(work["tokens_layers"], world, ems), "unit": UNIT,
                "ms_per_step": ems,
                "h2d_bytes_per_step": int(Q.numel() * Q.element_size() + K.numel() * K.element_size()
                                          + V.numel() * V.element_size()),

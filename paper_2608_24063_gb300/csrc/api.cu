@@ -57,13 +57,15 @@ struct Layout {
   int units_fuse_tc = 0, units_gather = 0;
   int64_t vs_rows = 0;
   int max_n = 0;
+  int64_t total_chunks = 0;
+  int max_chunks = 0;
   // derived sizes
   int64_t lse_elems = 0, score_elems = 0, out_rows = 0, drop_rows = 0;
   int units_lse = 0, units_col = 0, units_fuse = 0;
   // workspace offsets
   size_t o_status = 0, o_req = 0, o_layer = 0, o_u_lse = 0, o_u_col = 0, o_u_fuse = 0,
          o_row0 = 0, o_u_tc1 = 0, o_u_tc2 = 0, o_u_fuse_tc = 0, o_u_gather = 0, o_vs = 0, table_begin = 0, table_end = 0, o_lse = 0,
-         o_part = 0, o_lsep = 0, o_scores = 0, o_keys = 0, o_vals = 0, o_rank = 0, o_drop = 0, total = 0;
+         o_part = 0, o_lsep = 0, o_scores = 0, o_chunks = 0, o_rank = 0, o_drop = 0, total = 0;
   // host images
   std::vector<Req> req;
   std::vector<Layer> layer;
@@ -84,6 +86,8 @@ struct Layout {
     u_gather.assign((size_t)n_req * L + 1, 0);
     vs_rows = 0;
     max_n = 0;
+    total_chunks = 0;
+    max_chunks = 0;
     u_tc2.assign(n_req + 1, 0);
     base_tc1.assign(n_req, 0);
     q_rows = k_rows = max_rows = prows = max_prows = 0;
@@ -107,6 +111,12 @@ struct Layout {
       q.lsep_off = prows;
       q.vs_row0 = vs_rows;
       max_n = std::max(max_n, p.n);
+      {
+        const int chunks = (p.n + kSortChunk - 1) / kSortChunk;
+        q.chunk0 = (int32_t)total_chunks;
+        total_chunks += (int64_t)per_req_problems * chunks;
+        max_chunks = std::max(max_chunks, chunks);
+      }
       prows += (int64_t)L * Hkv * q.C * 128;
       max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
       q.nrb = (G * p.W + 255) / 256;
@@ -169,8 +179,7 @@ struct Layout {
     }
     if (need_scores) o_scores = a.take(sizeof(float) * score_elems);
     if (need_sort) {
-      o_keys = a.take(sizeof(uint32_t) * 2 * score_elems);
-      o_vals = a.take(sizeof(int32_t) * 2 * score_elems);
+      o_chunks = a.take(sizeof(uint64_t) * kSortChunk * std::max<int64_t>(total_chunks, 1));
       if (need_scores) o_rank = a.take(sizeof(int32_t) * score_elems);
     }
     if (need_drop) o_drop = a.take(sizeof(int32_t) * drop_rows);
@@ -447,9 +456,8 @@ int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis, c
   cudaError_t e = lay.upload(w, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
   const int problems = rank_mode == VC_RANK_PER_LAYER ? L * Hkv : Hkv;
-  e = launch_select(lay.shape(1.f), lay.tables(w), problems, lay.max_n, scores, rank_out,
-                    reinterpret_cast<uint32_t*>(w + lay.o_keys),
-                    reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, keep_idx,
+  e = launch_select(lay.shape(1.f), lay.tables(w), problems, lay.max_chunks, scores, rank_out,
+                    reinterpret_cast<uint64_t*>(w + lay.o_chunks), keep_idx,
                     drop_idx, st);
   return cuda_status(e);
 }
@@ -512,8 +520,8 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw, 
   const Shape sh = lay.shape(scale);
   const Tables tb = lay.tables(w);
   const int problems = lay.n_req * (p->rank_mode == VC_RANK_PER_LAYER ? p->L * p->Hkv : p->Hkv);
-  e = launch_select(sh, tb, problems, lay.max_n, scores, rank, reinterpret_cast<uint32_t*>(w + lay.o_keys),
-                    reinterpret_cast<int32_t*>(w + lay.o_vals), lay.score_elems, idx_out, drop, st);
+  e = launch_select(sh, tb, problems, lay.max_chunks, scores, rank,
+                    reinterpret_cast<uint64_t*>(w + lay.o_chunks), idx_out, drop, st);
   if (e != cudaSuccess) return VC_ERR_CUDA;
   e = launch_fuse(p->dtype, K, V, lay, sh, tb, idx_out, drop, p->mu, p->tau, K_out, V_out, w, st);
   return cuda_status(e);

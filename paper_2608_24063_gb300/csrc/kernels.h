@@ -49,11 +49,12 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
                            void* K_out, void* V_out, void* Vs, int64_t vs_rows, int units_gather,
                            int units, cudaStream_t st);
 
-// Ranking (radix sort per problem) and ascending keep/drop compaction.
-cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int max_n,
-                          const float* scores, int32_t* rank, uint32_t* keys, int32_t* vals,
-                          int64_t sort_stride, int32_t* keep_idx, int32_t* drop_idx,
-                          cudaStream_t st);
+// Ranking (sorted 1024-key chunks, `chunks`: kSortChunk keys per chunk,
+// Req::chunk0 locates a request's chunks) and ascending keep/drop compaction.
+constexpr int kSortChunk = 1024;
+cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int max_chunks,
+                          const float* scores, int32_t* rank, uint64_t* chunks, int32_t* keep_idx,
+                          int32_t* drop_idx, cudaStream_t st);
 
 // K_out = K[keep] (bit-exact), total_rows = Hkv * sum over requests and layers of B_l.
 cudaError_t launch_gather_k(int dtype, const void* K, const Shape& sh, const Tables& tb,

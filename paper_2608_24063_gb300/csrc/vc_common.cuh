@@ -27,7 +27,7 @@ struct Req {                 // one request of a batch
                              // whole 256-row chunks: 2*ceil(G*W/256)
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
   int32_t tiles;             // 256-key tiles, ceil(n/256)
-  int32_t pad_;
+  int32_t chunk0;            // first 1024-key sort chunk of its first ranking problem
 };
 
 struct Layer {               // one (request, layer)

@@ -75,6 +75,9 @@ def test_entry_points_reject_bad_arguments_without_touching_the_device():
     # workspace too small / misaligned
     assert lib.prunekv_score(p, p, 0, 1, 2, 1, 64, 10, 4, 0.0, 0, None, p, p, 16, None) == vc.VC_ERR_WORKSPACE
     assert lib.prunekv_score(p, p, 0, 1, 2, 1, 64, 10, 4, 0.0, 0, None, p, ctypes.c_void_p(272), 1 << 20, None) == vc.VC_ERR_WORKSPACE
+    # more tokens than the documented maximum
+    B1 = (ctypes.c_int32 * 1)(3)
+    assert lib.prunekv_select(p, 1, 1, 65537, B1, 4, 0, p, p, p, p, 1 << 30, None) == vc.VC_ERR_INVALID_ARG
     # B_l > Nq, Nq > n
     B = (ctypes.c_int32 * 2)(5, 3)
     assert lib.prunekv_select(p, 2, 1, 10, B, 4, 0, p, p, p, p, 1 << 20, None) == vc.VC_ERR_INVALID_ARG
@@ -92,7 +95,10 @@ def test_entry_points_reject_bad_arguments_without_touching_the_device():
 def test_workspace_sizes_are_positive_and_aligned():
     assert vc.prunekv_score_workspace_size(28, 28, 64) % 256 == 0
     assert vc.prunekv_score_workspace_size(28, 28, 64) >= 28 * 28 * 64 * 4
-    assert vc.prunekv_select_workspace_size(28, 4, 12544) >= 2 * 8 * 4 * 12544
+    # sorted 1024-key chunks (8-byte keys) for every ranking problem
+    assert vc.prunekv_select_workspace_size(28, 4, 12544) >= 8 * 1024 * 4 * 13
+    assert vc.prunekv_select_workspace_size(28, 4, 12544, vc.VC_RANK_PER_LAYER) >= 8 * 1024 * 28 * 4 * 13
+    assert vc.prunekv_select_workspace_size(2, 2, 65536) >= 8 * 65536 * 2
     assert vc.prunekv_fuse_workspace_size([3833, 1916], 4, 128, 12544, 4237) > 4 * 4237 * 2 * 256
     b = vc.Batch([12544], [64], [(19, 100)])
     prm = vc.make_params(28, 28, 4, 128, vc.VC_BF16)

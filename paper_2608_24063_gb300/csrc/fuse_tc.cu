@@ -64,47 +64,51 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
 //
 // A pair owns 256 kept rows of one (request, layer, KV head) (CTA r: rows
 // r*128 ... r*128+127, one per TMEM lane) and streams the dropped rows in
-// tiles of 128.  Per tile j the even CTA issues
-//   S = V_k V_d(j)^T   2-SM MMA, M = 256, N = 128 dropped rows (CTA r stages
-//                      dropped rows r*64 ... r*64+63, K-major),
-//   O += P(j) V_d(j)   2-SM MMA, M = 256, N = 128 value columns (CTA r stages
-//                      columns r*64 ... r*64+63 of all 128 dropped rows,
-//                      MN-major), A = P read from tensor memory,
-// in the order S(0), [P(0) ready] O(0), S(1), [P(1) ready] O(1), ...  P(j) is
-// written in bf16 over the first half of each softmax warp's own S columns,
-// so S(j+1) (issued after O(j)) may reuse them.  Two pairs run per TPC, so
-// one pair's softmax and prologue overlap the other's MMAs.
+// tiles of 64.  Per tile j the even CTA issues
+//   S(j) = V_k V_d(j)^T  2-SM MMA, M = 256, N = 64 dropped rows (CTA r stages
+//                        dropped rows r*32 ... r*32+31, K-major),
+//   O += P(j) V_d(j)     2-SM MMA, M = 256, N = 128 value columns, K = 64 (CTA
+//                        r stages columns r*64 ... of all 64 dropped rows,
+//                        MN-major), A = P read from tensor memory,
+// in the order S(0), S(1), [P(0)] O(0), S(2), [P(1)] O(1), ...: S is double
+// buffered, so S(j+1) is computed while the softmax works on tile j.  P(j) is
+// written in bf16 over the first half of each softmax warp's own S(j)
+// columns; S(j+2) reuses the buffer only after O(j) (issued before it) has
+// read P(j).  Two pairs run per TPC, so one pair's prologue and epilogue
+// overlap the other's work.
 //
-// Tensor memory per CTA (256 columns): O in [0, 128), S / P in [128, 256).
-// Softmax: warps w and w+4 share the TMEM lanes of warp w % 4; warp w takes
-// S columns 0-63 (dropped rows 0-63 of the tile), warp w+4 columns 64-127.
-// They agree on the row's reference maximum through shared memory each
-// tile; the maximum is raised (and O rescaled in tensor memory) only when a
-// tile exceeds it by more than 2^8.
+// Tensor memory per CTA (256 columns): O in [0, 128), S/P buffer b in
+// [128 + 64b, 192 + 64b).  Softmax: warps w and w+4 share the TMEM lanes of
+// warp w % 4; warp w takes S columns 0-31 (dropped rows 0-31 of the tile), warp
+// w+4 columns 32-63.  They agree on the row's reference maximum through shared
+// memory each tile; the maximum is raised (and O rescaled in tensor memory,
+// after O(j-1) is done) only when a tile exceeds it by more than 2^8.
 
 constexpr int kThreads = 320;
 constexpr int kProducerWarp = 8, kMmaWarp = 9;
-constexpr uint32_t kTile = 128;
+constexpr uint32_t kTile = 128;                  // kept rows per CTA
 constexpr uint32_t kKB = kTile * 128;            // 128 rows x 128 bytes
-constexpr uint32_t kHalfKB = 64 * 128;           // 64 rows x 128 bytes
-constexpr int kVdStages = 2;
-constexpr uint32_t kTmemCols = 256;              // O: [0,128), S/P: [128,256)
+constexpr uint32_t kDTile = 64;                  // dropped rows per tile (both CTAs)
+constexpr uint32_t kDHalfKB = 32 * 128;          // 32 rows x 128 bytes
+constexpr uint32_t kDKB = kDTile * 128;          // 64 rows x 128 bytes
+constexpr int kVdStages = 4;
+constexpr uint32_t kTmemCols = 256;              // O: [0,128), S/P buffers: [128,192), [192,256)
 constexpr uint32_t kSCol = 128;
 constexpr float kRescaleLog2 = 8.f;
 
 struct FSmem {
-  uint8_t vk[2][kKB];                 // this CTA's 128 kept rows [K-block]: A of S = V_k V_d^T
-  uint8_t vds[kVdStages][2][kHalfKB]; // this CTA's 64 dropped rows [stage][K-block]: B of S
-  uint8_t vdo[kVdStages][kKB];        // all 128 dropped rows, this CTA's 64 columns: B of O += P V_d
-  float xmax[2][4][2][32];            // [tile & 1][lane quadrant][column half][lane]: tile maxima
-  float lsum[2][4][32];               // [column half][lane quadrant][lane]: partial row sums
-  uint64_t vk_own;                    // this CTA's kept rows landed
-  uint64_t vk_pair;                   // even CTA: both CTAs' kept rows landed (2 arrivals)
-  uint64_t vd_full[kVdStages];        // even CTA: both CTAs' dropped tiles landed
-  uint64_t vd_empty[kVdStages];       // both: the MMAs reading the stage are done
-  uint64_t s_full;                    // both: S(j) is in tensor memory (and O(j-1) done)
-  uint64_t p_full;                    // even CTA: all 16 softmax warps wrote P(j)
-  uint64_t o_full;                    // both: the last O product is done
+  uint8_t vk[2][kKB];                  // this CTA's 128 kept rows [K-block]: A of S = V_k V_d^T
+  uint8_t vdo[kVdStages][kDKB];        // all 64 dropped rows, this CTA's 64 columns: B of O += P V_d
+  uint8_t vds[kVdStages][2][kDHalfKB]; // this CTA's 32 dropped rows [stage][K-block]: B of S
+  float xmax[2][4][2][32];             // [tile & 1][lane quadrant][column half][lane]: tile maxima
+  float lsum[2][4][32];                // [column half][lane quadrant][lane]: partial row sums
+  uint64_t vk_own;                     // this CTA's kept rows landed
+  uint64_t vk_pair;                    // even CTA: both CTAs' kept rows landed (2 arrivals)
+  uint64_t vd_full[kVdStages];         // even CTA: both CTAs' dropped tiles landed
+  uint64_t vd_empty[kVdStages];        // both: the MMAs reading the stage are done
+  uint64_t s_full[2];                  // both: S(j) is in S/P buffer j % 2
+  uint64_t p_full;                     // even CTA: all 16 softmax warps wrote P(j)
+  uint64_t o_done;                     // both: O(j) is done (phase j)
   uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
@@ -138,7 +142,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 2)
 fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_constant__ CUtensorMap tmRows64,
-                 Shape sh, Tables tb, float mu, float c2, __nv_bfloat16* __restrict__ V_out) {
+                 const __grid_constant__ CUtensorMap tmRows32, Shape sh, Tables tb, float mu, float c2,
+                 __nv_bfloat16* __restrict__ V_out) {
   extern __shared__ uint8_t smem_raw[];
   FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -155,7 +160,7 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
   const int r0 = (u % ktiles) * 2 * (int)kTile + (int)rank * (int)kTile;   // this CTA's first kept row
   const int rows = max(0, min((int)kTile, ly.B - r0));                    // kept rows of this CTA
   const int D = ly.D;
-  const int nt = (D + (int)kTile - 1) / (int)kTile;
+  const int nt = (D + (int)kDTile - 1) / (int)kDTile;
   // rows of this (layer, KV head) in Vs: B kept, then D dropped
   const int vs0 = (int)(rq.vs_row0 + (int64_t)sh.Hkv * (ly.P + ly.Qd) + (int64_t)g * (ly.B + D));
   const int64_t orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
@@ -164,9 +169,10 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     mbar_init(&sm.vk_own, 1);
     mbar_init(&sm.vk_pair, 2);
     for (int i = 0; i < kVdStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
-    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.s_full[0], 1);
+    mbar_init(&sm.s_full[1], 1);
     mbar_init(&sm.p_full, 16);
-    mbar_init(&sm.o_full, 1);
+    mbar_init(&sm.o_done, 1);
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
     fence_mbar_init();
@@ -186,6 +192,7 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     // ---- TMA producer (both CTAs)
     prefetch_tmap(&tmRows128);
     prefetch_tmap(&tmRows64);
+    prefetch_tmap(&tmRows32);
     mbar_arrive_expect_tx(&sm.vk_own, 2 * kKB);
     for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.vk[kb], &tmRows128, kb * 64, vs0 + r0, &sm.vk_own);
     int issued = 0;
@@ -198,12 +205,12 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       }
       const int st = j % kVdStages;
       if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
-      if (rank == 0) mbar_arrive_expect_tx(&sm.vd_full[st], 2 * (2 * kHalfKB + kKB));
+      if (rank == 0) mbar_arrive_expect_tx(&sm.vd_full[st], 2 * (2 * kDHalfKB + kDKB));
       const uint32_t full0 = map_to_rank(smem_u32(&sm.vd_full[st]), 0);
-      const int y = vs0 + ly.B + j * (int)kTile;
-      tma_load_2d_pair(sm.vds[st][0], &tmRows64, 0, y + (int)rank * 64, full0);
-      tma_load_2d_pair(sm.vds[st][1], &tmRows64, 64, y + (int)rank * 64, full0);
-      tma_load_2d_pair(sm.vdo[st], &tmRows128, (int)rank * 64, y, full0);
+      const int y = vs0 + ly.B + j * (int)kDTile;
+      tma_load_2d_pair(sm.vds[st][0], &tmRows32, 0, y + (int)rank * 32, full0);
+      tma_load_2d_pair(sm.vds[st][1], &tmRows32, 64, y + (int)rank * 32, full0);
+      tma_load_2d_pair(sm.vdo[st], &tmRows64, (int)rank * 64, y, full0);
       ++issued;
     }
     if (nt <= kVdStages && mbar_wait(&sm.vk_own, 0, abort))
@@ -212,41 +219,43 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       for (int i = max(0, issued - kVdStages); i < issued; ++i)
         drain_wait(&sm.vd_full[i % kVdStages], (i / kVdStages) & 1);
   } else if (warp == kMmaWarp && lane == 0 && rank == 0 && nt > 0) {
-    // ---- MMA issuer (even CTA)
-    const uint32_t id_s = idesc_bf16_f32(2 * kTile, kTile);
+    // ---- MMA issuer (even CTA): S(0), S(1), O(0), S(2), O(1), ...
+    const uint32_t id_s = idesc_bf16_f32(2 * kTile, kDTile);
     const uint32_t id_o = idesc_bf16_f32_bmn(2 * kTile, kTile);
-    const uint32_t s_tm = tbase + kSCol;
     bool ok = mbar_wait(&sm.vk_pair, 0, abort);
-    int jo = 0;                                   // next O product to issue
+    int jo = 0;                                   // O products issued
     for (int j = 0; ok && j <= nt; ++j) {
-      if (j >= 1) {
-        // O += P(j-1) V_d(j-1), once the softmax has written P(j-1)
-        if (!mbar_wait(&sm.p_full, (j - 1) & 1, abort)) break;
-        tc_fence_after();
-        const int st = (j - 1) % kVdStages;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_pair_ta(tbase, s_tm + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
-                           desc_sw128_mn(smem_u32(sm.vdo[st]) + kk * 2048, kKB), id_o,
-                           (j > 1 || kk > 0) ? 1u : 0u);
-        mma_commit_pair(&sm.vd_empty[st], 3);
-        jo = j;
-      }
       if (j < nt) {
-        // S(j) = V_k V_d(j)^T (after O(j-1) in the pipe, so P(j-1) has been read)
+        // S(j) into buffer j % 2 (its previous user O(j-2) was issued before)
         const int st = j % kVdStages;
         if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
         tc_fence_after();
+        const uint32_t s_tm = tbase + kSCol + (uint32_t)(j & 1) * kDTile;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           mma_bf16_pair(s_tm, desc_sw128(smem_u32(sm.vk[kk >> 2]) + (kk & 3) * 32),
                         desc_sw128(smem_u32(sm.vds[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
-        mma_commit_pair(&sm.s_full, 3);
+        mma_commit_pair(&sm.s_full[j & 1], 3);
+      }
+      if (j >= 1) {
+        // O += P(j-1) V_d(j-1), once the softmax has written P(j-1)
+        const int jp = j - 1, st = jp % kVdStages;
+        if (!mbar_wait(&sm.p_full, jp & 1, abort)) break;
+        tc_fence_after();
+        const uint32_t p_tm = tbase + kSCol + (uint32_t)(jp & 1) * kDTile;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_bf16_pair_ta(tbase, p_tm + (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8),
+                           desc_sw128_mn(smem_u32(sm.vdo[st]) + kk * 2048, kDKB), id_o,
+                           (jp > 0 || kk > 0) ? 1u : 0u);
+        mma_commit_pair(&sm.vd_empty[st], 3);
+        mma_commit_pair(&sm.o_done, 3);
+        jo = j;
       }
     }
-    if (jo == nt) mma_commit_pair(&sm.o_full, 3);
     mma_commit_pair(&sm.mma_done, 1);
     drain_wait(&sm.mma_done, 0);
+    (void)jo;
   } else if (warp < 8) {
     // ---- softmax over the drop set and epilogue: one kept row per TMEM lane
     const int q4 = warp & 3;                          // lane quadrant
@@ -254,72 +263,72 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     const int row = (q4 << 5) + lane;                 // row within this CTA's 128
     const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
     const uint32_t o_col = tbase + lane_off + (uint32_t)hf * 64;
-    const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)hf * 64;
     const uint32_t p_full0 = lane == 0 ? map_to_rank(smem_u32(&sm.p_full), 0) : 0u;
     float m = -INFINITY, lsum = 0.f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      if (!warp_wait(&sm.s_full, j & 1, abort)) { ok = false; break; }
+      const int bsel = j & 1;
+      if (!warp_wait(&sm.s_full[bsel], (j >> 1) & 1, abort)) { ok = false; break; }
       tc_fence_after();
-      float x[4][16];
+      // this warp's 32 columns of S(j)
+      const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)bsel * kDTile + (uint32_t)hf * 32;
+      float x[2][16];
       {
-        uint32_t v[4][16];
+        uint32_t v[2][16];
 #pragma unroll
-        for (int p = 0; p < 4; ++p) tmem_ld16(s_col + p * 16, v[p]);
+        for (int p = 0; p < 2; ++p) tmem_ld16(s_col + p * 16, v[p]);
         tmem_wait_only();
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
+        for (int p = 0; p < 2; ++p) {
           reg_fence(v[p]);
 #pragma unroll
           for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
         }
       }
-      const int valid = min(64, D - j * (int)kTile - hf * 64);
-      if (valid < 64) {                               // last tile: columns past D
+      const int valid = min(32, D - j * (int)kDTile - hf * 32);
+      if (valid < 32) {                               // last tile: columns past D
 #pragma unroll
-        for (int p = 0; p < 4; ++p)
+        for (int p = 0; p < 2; ++p)
 #pragma unroll
           for (int q = 0; q < 16; ++q)
             if (p * 16 + q >= valid) x[p][q] = -INFINITY;
       }
       float a0 = fmaxf(x[0][0], x[0][1]), a1 = fmaxf(x[1][0], x[1][1]);
-      float a2 = fmaxf(x[2][0], x[2][1]), a3 = fmaxf(x[3][0], x[3][1]);
 #pragma unroll
       for (int q = 2; q < 16; q += 2) {
         a0 = fmax3(a0, x[0][q], x[0][q + 1]);
         a1 = fmax3(a1, x[1][q], x[1][q + 1]);
-        a2 = fmax3(a2, x[2][q], x[2][q + 1]);
-        a3 = fmax3(a3, x[3][q], x[3][q + 1]);
       }
       // this row's tile maximum over both column halves
-      sm.xmax[j & 1][q4][hf][lane] = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
+      sm.xmax[bsel][q4][hf][lane] = fmaxf(a0, a1);
       named_sync(1 + q4, 64);
-      const float tm = fmaxf(sm.xmax[j & 1][q4][0][lane], sm.xmax[j & 1][q4][1][lane]) * c2;
+      const float tm = fmaxf(sm.xmax[bsel][q4][0][lane], sm.xmax[bsel][q4][1][lane]) * c2;
       const bool raise = tm > m + kRescaleLog2;
       const float m_new = raise ? tm : m;
       const float corr = raise ? ex2(m - m_new) : 1.f;   // 0 on the first tile
       lsum *= corr;
       m = m_new;
-      // P = exp2(S * c2 - m) in bf16 over the first 32 of this warp's S columns
+      // P = exp2(S * c2 - m) in bf16 over the first 16 of this warp's S columns
       const float2 sc = make_float2(c2, c2), nm = make_float2(-m, -m);
       float2 ls = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int hp = 0; hp < 2; ++hp) {
+      {
         uint32_t w[16];
 #pragma unroll
         for (int q = 0; q < 16; ++q) {
-          const int c = hp * 32 + 2 * q;
+          const int c = 2 * q;
           const float2 t = __ffma2_rn(make_float2(x[c >> 4][c & 15], x[c >> 4][(c & 15) + 1]), sc, nm);
           const float2 e = make_float2(ex2(t.x), ex2(t.y));
           ls = __fadd2_rn(ls, e);
           w[q] = pack_bf16x2(e.x, e.y);
         }
-        tmem_st16(s_col + hp * 16, w);
+        tmem_st16(s_col, w);
       }
       lsum += ls.x + ls.y;
       if (__any_sync(0xffffffffu, raise && j > 0)) {
-        // rare: O(j-1) is complete (S(j) was issued after it) and O(j) waits
-        // for P(j); rescale this warp's 64 columns of O in tensor memory
+        // rare: rescale this warp's 64 columns of O in tensor memory once
+        // O(j-1) is done (O(j) waits for P(j), so nothing else writes O)
+        if (!warp_wait(&sm.o_done, (j - 1) & 1, abort)) { ok = false; break; }
+        tc_fence_after();
 #pragma unroll 1
         for (int p = 0; p < 4; ++p) {
           uint32_t v[16];
@@ -338,15 +347,16 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped
     sm.lsum[hf][q4][lane] = lsum;
     const bool have_k = warp_wait(&sm.vk_own, 0, abort);
-    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_full, 0, abort);
+    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_done, (nt - 1) & 1, abort);
     __syncwarp();
     named_sync(5, 256);
     const float lt = sm.lsum[0][q4][lane] + sm.lsum[1][q4][lane];   // same order in both halves
     if (have_o) tc_fence_after();
     const float w_o = have_o ? (1.f - mu) / lt : 0.f;
     const float w_k = have_o ? mu : 1.f;
-    // stage the 128 x 128 output tile in the (now idle) dropped-row buffers:
-    // row r at r * 256 bytes, 16-byte chunk c at slot c ^ (r & 15)
+    // stage the 128 x 128 output tile in the (now idle) dropped-row buffers
+    // (vdo, 4 x 8 KB contiguous): row r at r * 256 bytes, 16-byte chunk c at
+    // slot c ^ (r & 15)
     uint8_t* stage = &sm.vdo[0][0];
 #pragma unroll 1
     for (int hh = 0; hh < 2; ++hh) {                  // 32 of this warp's 64 columns at a time
@@ -456,15 +466,16 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  CUtensorMap m128, m64;
-  if (!make_rows_map(&m128, Vs, (uint64_t)vs_rows, kTile) || !make_rows_map(&m64, Vs, (uint64_t)vs_rows, 64))
+  CUtensorMap m128, m64, m32;
+  if (!make_rows_map(&m128, Vs, (uint64_t)vs_rows, kTile) || !make_rows_map(&m64, Vs, (uint64_t)vs_rows, 64) ||
+      !make_rows_map(&m32, Vs, (uint64_t)vs_rows, 32))
     return cudaErrorInvalidValue;
   const size_t smem = sizeof(FSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(fuse_v_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   ProfileScope ps("fuse_v_tc", st);
-  fuse_v_tc_kernel<<<2 * units, kThreads, smem, st>>>(m128, m64, sh, tb, mu, kLog2e / tau,
+  fuse_v_tc_kernel<<<2 * units, kThreads, smem, st>>>(m128, m64, m32, sh, tb, mu, kLog2e / tau,
                                                       static_cast<__nv_bfloat16*>(V_out));
   return cudaGetLastError();
 }

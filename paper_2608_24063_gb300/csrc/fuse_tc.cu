@@ -30,9 +30,13 @@ using namespace tc;
 // ---------------------------------------------------------------------------
 // survivor gather
 
-constexpr int kGatherThreads = 256;   // 16 rows x 16 chunks of 16 bytes
-constexpr int kGatherRows = 16;
+constexpr int kGatherThreads = 256;   // 16 row slots x 16 chunks of 16 bytes
+constexpr int kGatherRowsPerThread = 4;
+constexpr int kGatherRows = 16 * kGatherRowsPerThread;   // rows per block
 
+// Each thread copies its 16-byte chunk of four rows (i, i+16, i+32, i+48 of
+// the block), all index loads and then all row loads in flight before the
+// stores, so the dependent loads overlap.
 __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
     const uint4* __restrict__ K, const uint4* __restrict__ V, Shape sh, Tables tb,
     const int32_t* __restrict__ keep_idx, const int32_t* __restrict__ drop_idx,
@@ -45,18 +49,40 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
   const int blocks = (nsurv + kGatherRows - 1) / kGatherRows;
   const int u = blockIdx.x - tb.unit0_gather[rl];
   const int g = u / blocks;
-  const int i = (u % blocks) * kGatherRows + (threadIdx.x >> 4);
+  const int i0 = (u % blocks) * kGatherRows + (threadIdx.x >> 4);
   const int c = threadIdx.x & 15;
-  if (i >= nsurv) return;
-  const int32_t v = i < ly.B ? keep_idx[rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + i]
-                             : drop_idx[rq.drop_row0 + (int64_t)sh.Hkv * ly.Qd + (int64_t)g * ly.D + (i - ly.B)];
-  if (v < 0 || v >= rq.n) {
-    if (c == 0) set_status(tb.status, VC_ERR_DEVICE_INDEX);
-    return;
+  const int64_t kbase = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B;
+  const int64_t dbase = rq.drop_row0 + (int64_t)sh.Hkv * ly.Qd + (int64_t)g * ly.D;
+  const int64_t sbase = rq.vs_row0 + (int64_t)sh.Hkv * (ly.P + ly.Qd) + (int64_t)g * nsurv;
+  const int64_t src0 = (rq.kv_off / 8) + ((int64_t)l * sh.Hkv + g) * rq.n * 16 + c;
+  int32_t v[kGatherRowsPerThread];
+#pragma unroll
+  for (int k = 0; k < kGatherRowsPerThread; ++k) {
+    const int i = i0 + 16 * k;
+    v[k] = -1;
+    if (i < nsurv) {
+      const int32_t t = i < ly.B ? keep_idx[kbase + i] : drop_idx[dbase + (i - ly.B)];
+      if (t >= 0 && t < rq.n) v[k] = t;
+      else if (c == 0) set_status(tb.status, VC_ERR_DEVICE_INDEX);
+    }
   }
-  const int64_t src = (rq.kv_off / 8) + (((int64_t)l * sh.Hkv + g) * rq.n + v) * 16 + c;
-  Vs[(rq.vs_row0 + (int64_t)sh.Hkv * (ly.P + ly.Qd) + (int64_t)g * nsurv + i) * 16 + c] = V[src];
-  if (i < ly.B) K_out[(rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + i) * 16 + c] = K[src];
+  uint4 vv[kGatherRowsPerThread], kv[kGatherRowsPerThread];
+#pragma unroll
+  for (int k = 0; k < kGatherRowsPerThread; ++k) {
+    if (v[k] >= 0) {
+      const int64_t src = src0 + (int64_t)v[k] * 16;
+      vv[k] = V[src];
+      if (i0 + 16 * k < ly.B) kv[k] = K[src];
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kGatherRowsPerThread; ++k) {
+    const int i = i0 + 16 * k;
+    if (v[k] >= 0) {
+      Vs[(sbase + i) * 16 + c] = vv[k];
+      if (i < ly.B) K_out[(kbase + i) * 16 + c] = kv[k];
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------

@@ -70,7 +70,7 @@ def plans_for(wl, vc):
 
 def algorithmic(wl, plans):
     eb = 2 if wl.dtype == "bf16" else 4
-    tot = dict(bytes=0, flops_score=0, flops_fuse=0, k_bytes=0, gather_bytes=0, fuse_bytes=0,
+    tot = dict(bytes=0, flops_score=0, flops_fuse=0, k_bytes=0, gather_bytes=0, fuse_bytes=0, surv_v_bytes=0,
                tokens_layers=0)
     for r, (B, Nq, h) in zip(wl.requests, plans):
         T = sum(B)
@@ -84,6 +84,7 @@ def algorithmic(wl, plans):
         tot["k_bytes"] += k_all + q
         tot["gather_bytes"] += 2 * kept_k
         tot["fuse_bytes"] += surv_v + wl.Hkv * T * row
+        tot["surv_v_bytes"] += surv_v
         tot["flops_score"] += 2 * wl.Hq * r.W * r.n * wl.d * wl.L
         tot["flops_fuse"] += 4 * wl.Hkv * wl.d * sum(b * (Nq - b) for b in B if b > 0)
         tot["tokens_layers"] += r.n * wl.L
@@ -412,6 +413,9 @@ def main():
         dKo = [K_out, torch.empty_like(K_out)]
         dVo = [V_out, torch.empty_like(V_out)]
         dI = [idx, torch.empty_like(idx)]
+        # V can stay in pinned host memory when the device reads it directly:
+        # only the survivors' rows then cross to the GPU (read by the gather)
+        v_host = all(vc.viscache_device_accessible(t) for t in hV)
         s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         ev = lambda: torch.cuda.Event()
         in_done, cmp_done, out_done = [ev(), ev()], [ev(), ev()], [ev(), ev()]
@@ -423,13 +427,14 @@ def main():
             with torch.cuda.stream(s_in):
                 dQ[bsel].copy_(hQ[bsel], non_blocking=True)
                 dK[bsel].copy_(hK[bsel], non_blocking=True)
-                dV[bsel].copy_(hV[bsel], non_blocking=True)
+                if not v_host:
+                    dV[bsel].copy_(hV[bsel], non_blocking=True)
                 in_done[bsel].record(s_in)
             s_cmp.wait_event(in_done[bsel])
             if i >= 2:
                 s_cmp.wait_event(out_done[bsel])       # step i-2's outputs are back on the host
-            vc.prunekv_compress(batch, prm, dQ[bsel], dK[bsel], dV[bsel], dKo[bsel], dVo[bsel], dI[bsel],
-                                ws, stream=s_cmp)
+            vc.prunekv_compress(batch, prm, dQ[bsel], dK[bsel], hV[bsel] if v_host else dV[bsel], dKo[bsel],
+                                dVo[bsel], dI[bsel], ws, stream=s_cmp)
             cmp_done[bsel].record(s_cmp)
             s_out.wait_event(cmp_done[bsel])
             with torch.cuda.stream(s_out):
@@ -455,10 +460,13 @@ def main():
         assert vc.prunekv_get_status(ws) == vc.VC_OK
         assert torch.equal(oI[(e_steps - 1) % 2], dI[(e_steps - 1) % 2].cpu())
         ems = max_over_ranks(a.elapsed_time(b) / e_steps, world, dist, dev)
+        v_bytes = work["surv_v_bytes"] if v_host else V.numel() * V.element_size()
         e2e = {"value": job_value(work["tokens_layers"], world, ems), "unit": UNIT,
                "ms_per_step": ems, "pipelined": "copy-in / compress / copy-out on three streams",
+               "v_source": "pinned host memory read by the gather kernel (survivor rows only)"
+                           if v_host else "copied to the device every step",
                "h2d_bytes_per_step": int(Q.numel() * Q.element_size() + K.numel() * K.element_size()
-                                         + V.numel() * V.element_size()),
+                                         + v_bytes),
                "d2h_bytes_per_step": int(K_out.numel() * K_out.element_size()
                                          + V_out.numel() * V_out.element_size()
                                          + idx.numel() * idx.element_size())}

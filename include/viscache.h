@@ -194,6 +194,10 @@ int prunekv_fuse_compact(const void* K, const void* V, int dtype, int32_t L, int
  * a single request:  K/V of request r start at element L*Hkv*d*sum_{r'<r} n_r',
  * Qw of request r at element L*Hq*d*sum_{r'<r} W_r'.  Outputs likewise: request
  * r's dense varlen cache starts at row Hkv * sum_{r'<r} T_r' (T_r = sum_l B_l).
+ * Qw, K, the outputs and ws are device memory.  V may also be host memory the
+ * device can read (viscache_device_accessible(V) == 1): only the rows of the
+ * surviving tokens of layers with B_l > 0 are read, once, so V can stay on the
+ * host while Qw and K are copied in.
  */
 typedef struct {
     int32_t n_req;            /* number of requests, >= 1 */
@@ -250,6 +254,16 @@ int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* lau
 #define VC_PATH_AUTO 0
 #define VC_PATH_SIMT 1
 int viscache_set_kernel_path(int path);
+
+/*
+ * viscache_device_accessible -- 1 if the current device can read `ptr`
+ * directly (device memory, managed memory, or host memory mapped into the
+ * device's address space, e.g. pinned with cudaHostAlloc under unified
+ * addressing), 0 if not, -VC_ERR_CUDA if the query fails.  Not a step of the
+ * pass: it tells a caller whether V may stay in host memory (see
+ * prunekv_compress).  No device work, no synchronisation.
+ */
+int viscache_device_accessible(const void* ptr);
 
 /* Version string of the library build. */
 const char* viscache_version(void);

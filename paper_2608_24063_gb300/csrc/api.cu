@@ -406,6 +406,18 @@ extern "C" {
 
 const char* viscache_version(void) { return "viscache-gb300 0.2 (sm_103a)"; }
 
+int viscache_device_accessible(const void* ptr) {
+  if (!ptr) return 0;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    cudaGetLastError();
+    return -VC_ERR_CUDA;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return 1;
+  if (a.type == cudaMemoryTypeHost) return a.devicePointer == ptr ? 1 : 0;
+  return 0;
+}
+
 int viscache_set_kernel_path(int path) {
   if (path != VC_PATH_AUTO && path != VC_PATH_SIMT) return VC_ERR_INVALID_ARG;
   g_path.store(path);

@@ -36,7 +36,8 @@ EXPORTED = ("viscache_plan_budgets", "prunekv_score_workspace_size", "prunekv_sc
             "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
-            "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path")
+            "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
+            "viscache_device_accessible")
 
 
 class VisCacheError(RuntimeError):
@@ -92,6 +93,7 @@ def lib() -> ctypes.CDLL:
         L.viscache_version.restype = ctypes.c_char_p
         L.viscache_profile_enable.argtypes = [i32]
         L.viscache_set_kernel_path.argtypes = [i32]
+        L.viscache_device_accessible.argtypes = [vp]
         L.viscache_profile_read.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(ctypes.c_float),
                                             pi32, i32]
         _lib = L
@@ -136,6 +138,14 @@ def _i32(seq):
 
 def viscache_version() -> str:
     return lib().viscache_version().decode()
+
+
+def viscache_device_accessible(t: torch.Tensor) -> bool:
+    """True if the current CUDA device can read the tensor's memory directly."""
+    rc = lib().viscache_device_accessible(ctypes.c_void_p(t.data_ptr()))
+    if rc < 0:
+        raise VisCacheError("viscache_device_accessible", -rc)
+    return rc == 1
 
 
 def viscache_plan_budgets(L: int, n_vis: int, rr_num: int, rr_den: int, h: int = 0,

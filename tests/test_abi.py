@@ -32,6 +32,10 @@ def test_version():
     assert "sm_103a" in vc.viscache_version()
 
 
+def test_device_accessible_null_pointer():
+    assert vc.lib().viscache_device_accessible(None) == 0
+
+
 @pytest.mark.parametrize("rr", [(19, 100), (22, 100), (23, 100), (28, 100), (1, 3), (56, 100)])
 def test_planner_matches_oracle_exhaustive_L(rr):
     for L in range(1, 129):

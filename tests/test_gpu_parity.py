@@ -261,6 +261,24 @@ def test_workload_full_parity(wid, kernel_path):
     assert torch.equal(idx, out["keep"]) and torch.equal(Ko, out["K_out"]) and torch.equal(Vo, out["V_out"])
 
 
+def test_values_in_host_memory(kernel_path):
+    # V may stay in pinned host memory the device can read: same bits as from HBM
+    L, Hq, Hkv, d, n, W = 4, 8, 2, 128, 1000, 32
+    Q = _rand((L, Hq, W, d), 9101, torch.bfloat16).to(DEV)
+    K = _rand((L, Hkv, n, d), 9102, torch.bfloat16).to(DEV)
+    V = _rand((L, Hkv, n, d), 9103, torch.bfloat16)
+    hV = V.pin_memory()
+    if not vc.viscache_device_accessible(hV):
+        pytest.skip("pinned host memory is not mapped into the device's address space here")
+    assert vc.viscache_device_accessible(K)
+    batch = vc.Batch([n], [W], [(19, 100)])
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    Ko1, Vo1, i1 = vc.prunekv_compress(batch, prm, Q, K, V.to(DEV))
+    Ko2, Vo2, i2 = vc.prunekv_compress(batch, prm, Q, K, hV)
+    torch.cuda.synchronize()
+    assert torch.equal(i1, i2) and torch.equal(Ko1, Ko2) and torch.equal(Vo1, Vo2)
+
+
 def test_generator_same_bits_on_device():
     wl = synth.scaled(synth.WORKLOADS[3], "slice", L=2)
     q_cpu = synth.make_q(wl, 0, "cpu")

@@ -133,9 +133,9 @@ struct FSmem {
   uint64_t vd_full[kVdStages];         // even CTA: both CTAs' dropped tiles landed
   uint64_t vd_empty[kVdStages];        // both: the MMAs reading the stage are done
   uint64_t s_full[2];                  // both: S(j) is in S/P buffer j % 2
-  uint64_t p_full;                     // even CTA: all 16 softmax warps wrote P(j)
+  uint64_t p_full[2];                  // even CTA: all 16 softmax warps wrote P(j), buffer j % 2
   uint64_t o_done;                     // both: O(j) is done (phase j)
-  uint64_t mma_done;
+  uint64_t mma_done;                   // both: every MMA of the pair is done (one phase)
   uint32_t tmem_base;
   int abort;
 };
@@ -197,7 +197,8 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     for (int i = 0; i < kVdStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
     mbar_init(&sm.s_full[0], 1);
     mbar_init(&sm.s_full[1], 1);
-    mbar_init(&sm.p_full, 16);
+    mbar_init(&sm.p_full[0], 16);
+    mbar_init(&sm.p_full[1], 16);
     mbar_init(&sm.o_done, 1);
     mbar_init(&sm.mma_done, 1);
     sm.abort = 0;
@@ -266,7 +267,7 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       if (j >= 1) {
         // O += P(j-1) V_d(j-1), once the softmax has written P(j-1)
         const int jp = j - 1, st = jp % kVdStages;
-        if (!mbar_wait(&sm.p_full, jp & 1, abort)) break;
+        if (!mbar_wait(&sm.p_full[jp & 1], (jp >> 1) & 1, abort)) break;
         tc_fence_after();
         const uint32_t p_tm = tbase + kSCol + (uint32_t)(jp & 1) * kDTile;
 #pragma unroll
@@ -279,7 +280,8 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
         jo = j;
       }
     }
-    mma_commit_pair(&sm.mma_done, 1);
+    // always committed (also after a give-up), so the epilogue's wait ends
+    mma_commit_pair(&sm.mma_done, 3);
     drain_wait(&sm.mma_done, 0);
     (void)jo;
   } else if (warp < 8) {
@@ -289,7 +291,6 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     const int row = (q4 << 5) + lane;                 // row within this CTA's 128
     const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
     const uint32_t o_col = tbase + lane_off + (uint32_t)hf * 64;
-    const uint32_t p_full0 = lane == 0 ? map_to_rank(smem_u32(&sm.p_full), 0) : 0u;
     float m = -INFINITY, lsum = 0.f;
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
@@ -352,7 +353,9 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       lsum += ls.x + ls.y;
       if (__any_sync(0xffffffffu, raise && j > 0)) {
         // rare: rescale this warp's 64 columns of O in tensor memory once
-        // O(j-1) is done (O(j) waits for P(j), so nothing else writes O)
+        // O(j-1) is done (O(j) waits for P(j), so nothing else writes O).  The
+        // parity wait is unambiguous: s_full(j) was committed after O(j-2), so
+        // o_done is in phase j-1 or j here.
         if (!warp_wait(&sm.o_done, (j - 1) & 1, abort)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll 1
@@ -368,12 +371,16 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(p_full0);
+      if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&sm.p_full[bsel]), 0));
     }
     // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped
     sm.lsum[hf][q4][lane] = lsum;
     const bool have_k = warp_wait(&sm.vk_own, 0, abort);
-    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.o_done, (nt - 1) & 1, abort);
+    // O is final once every MMA of the pair is done.  (A parity wait on o_done
+    // for O(nt-1) would be ambiguous here: s_full(nt-1) only guarantees O(nt-3),
+    // and with O(nt-2) still running the barrier sits in a phase of the other
+    // parity, which that wait would take as complete.)
+    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.mma_done, 0, abort);
     __syncwarp();
     named_sync(5, 256);
     const float lt = sm.lsum[0][q4][lane] + sm.lsum[1][q4][lane];   // same order in both halves

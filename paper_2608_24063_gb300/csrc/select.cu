@@ -13,6 +13,8 @@
 // block-wide scan over tokens in ascending position emits keep = {rank < B_l}
 // and drop = {B_l <= rank < Nq}, so both lists come out ascending and the
 // result does not depend on thread scheduling.
+#include <algorithm>
+
 #include "vc_common.cuh"
 #include "kernels.h"
 #include "profile.h"
@@ -48,6 +50,15 @@ __device__ __forceinline__ void problem_of(const Shape& sh, const Tables& tb, in
   chunk_base = ((int64_t)rq.chunk0 + (int64_t)k * nchunks) * kSortChunk;
 }
 
+// Compare-exchange of the bitonic network between lanes t and t ^ j of a
+// warp (j < 32): the lower lane keeps min/max as the direction bit says.
+__device__ __forceinline__ uint64_t bitonic_lane(uint64_t a, int t, int j, int k) {
+  const uint64_t b = __shfl_xor_sync(0xffffffffu, a, j);
+  const bool up = (t & k) == 0;
+  const bool lower = (t & j) == 0;
+  return (lower == up) ? (a < b ? a : b) : (a < b ? b : a);
+}
+
 __global__ void __launch_bounds__(kSortChunk) chunk_sort_kernel(Shape sh, Tables tb,
                                                                 const float* __restrict__ scores,
                                                                 uint64_t* __restrict__ chunks) {
@@ -60,26 +71,35 @@ __global__ void __launch_bounds__(kSortChunk) chunk_sort_kernel(Shape sh, Tables
   if (c >= nchunks) return;
   const int t = threadIdx.x;
   const int v = c * kSortChunk + t;
-  e[t] = v < rq.n ? ((uint64_t)desc_key(scores[off + v]) << 32) | (uint32_t)v : ~0ull;
+  uint64_t a = v < rq.n ? ((uint64_t)desc_key(scores[off + v]) << 32) | (uint32_t)v : ~0ull;
+  // strides below 32 stay in the warp (shuffles), larger ones go through
+  // shared memory with a block barrier
   for (int k = 2; k <= kSortChunk; k <<= 1) {
     for (int j = k >> 1; j > 0; j >>= 1) {
-      __syncthreads();
-      const int q = t ^ j;
-      if (q > t) {
-        const uint64_t a = e[t], b = e[q];
+      if (j >= 32) {
+        e[t] = a;
+        __syncthreads();
+        const uint64_t b = e[t ^ j];
         const bool up = (t & k) == 0;
-        if ((a > b) == up) { e[t] = b; e[q] = a; }
+        const bool lower = (t & j) == 0;
+        a = (lower == up) ? (a < b ? a : b) : (a < b ? b : a);
+        __syncthreads();
+      } else {
+        a = bitonic_lane(a, t, j, k);
       }
     }
   }
-  __syncthreads();
-  chunks[base + (int64_t)c * kSortChunk + t] = e[t];
+  chunks[base + (int64_t)c * kSortChunk + t] = a;
 }
+
+// Other chunks are staged kRankGroup at a time (8 KB each) so a group costs
+// one barrier pair; each thread then runs its binary searches back to back.
+constexpr int kRankGroup = 12;
 
 __global__ void __launch_bounds__(kSortChunk) chunk_rank_kernel(Shape sh, Tables tb,
                                                                 const uint64_t* __restrict__ chunks,
                                                                 int32_t* __restrict__ rank) {
-  __shared__ uint64_t other[kSortChunk];
+  extern __shared__ uint64_t other[];               // [kRankGroup][kSortChunk]
   Req rq;
   int64_t off, base;
   int nchunks;
@@ -89,16 +109,21 @@ __global__ void __launch_bounds__(kSortChunk) chunk_rank_kernel(Shape sh, Tables
   const int t = threadIdx.x;
   const uint64_t mine = chunks[base + (int64_t)c * kSortChunk + t];
   int count = t;                                   // elements of its own chunk below it
-  for (int c2 = 0; c2 < nchunks; ++c2) {
-    if (c2 == c) continue;
+  for (int g0 = 0; g0 < nchunks; g0 += kRankGroup) {
+    const int gn = min(kRankGroup, nchunks - g0);
     __syncthreads();
-    other[t] = chunks[base + (int64_t)c2 * kSortChunk + t];
+    for (int i = 0; i < gn; ++i)
+      other[i * kSortChunk + t] = chunks[base + (int64_t)(g0 + i) * kSortChunk + t];
     __syncthreads();
-    int pos = 0;                                   // elements of chunk c2 below `mine`
+    for (int i = 0; i < gn; ++i) {
+      if (g0 + i == c) continue;
+      const uint64_t* o = other + i * kSortChunk;
+      int pos = 0;                                 // elements of chunk g0 + i below `mine`
 #pragma unroll
-    for (int s = kSortChunk; s > 0; s >>= 1)
-      if (pos + s <= kSortChunk && other[pos + s - 1] < mine) pos += s;
-    count += pos;
+      for (int s = kSortChunk; s > 0; s >>= 1)
+        if (pos + s <= kSortChunk && o[pos + s - 1] < mine) pos += s;
+      count += pos;
+    }
   }
   if (mine != ~0ull) {
     const uint32_t v = (uint32_t)mine;
@@ -186,8 +211,11 @@ cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int
   cudaError_t e0 = cudaGetLastError();
   if (e0 != cudaSuccess) return e0;
   {
+    const size_t smem = sizeof(uint64_t) * kSortChunk * (size_t)std::min(kRankGroup, std::max(max_chunks, 1));
+    cudaError_t ea = cudaFuncSetAttribute(chunk_rank_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (ea != cudaSuccess) return ea;
     ProfileScope ps("chunk_rank", st);
-    chunk_rank_kernel<<<grid, kSortChunk, 0, st>>>(sh, tb, chunks, rank);
+    chunk_rank_kernel<<<grid, kSortChunk, smem, st>>>(sh, tb, chunks, rank);
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;

@@ -107,7 +107,8 @@ struct Layout {
       q.out_row0 = out_rows;
       q.drop_row0 = drop_rows;
       q.n = p.n; q.W = p.W; q.Nq = p.Nq; q.h = p.h;
-      q.C = 2 * ((G * p.W + 255) / 256);
+      q.C = (G * p.W + 255) / 256;
+      q.cw = 16 * ((G * p.W + 16 * q.C - 1) / (16 * q.C));
       q.lsep_off = prows;
       q.vs_row0 = vs_rows;
       max_n = std::max(max_n, p.n);
@@ -117,8 +118,8 @@ struct Layout {
         total_chunks += (int64_t)per_req_problems * chunks;
         max_chunks = std::max(max_chunks, chunks);
       }
-      prows += (int64_t)L * Hkv * q.C * 128;
-      max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * 128);
+      prows += (int64_t)L * Hkv * q.C * q.cw;
+      max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * q.cw);
       q.nrb = (G * p.W + 255) / 256;
       q.tiles = (p.n + 255) / 256;
       base_tc1[r] = L * Hkv * q.nrb;

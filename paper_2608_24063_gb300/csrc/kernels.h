@@ -32,7 +32,7 @@ struct TcPlan {
   int64_t q_rows;    // rows of the packed Qw tensor
   int64_t k_rows;    // rows of the packed K tensor
   int64_t max_rows;  // max over requests of L*Hq*W
-  int64_t max_prows; // max over requests of L*Hkv*C*128 (chunk-padded rows)
+  int64_t max_prows; // max over requests of L*Hkv*C*cw (chunk-padded rows)
 };
 int score_tc_max_splits();
 int score_tc_pair_slots();

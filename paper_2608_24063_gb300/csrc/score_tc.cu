@@ -220,6 +220,10 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     float m = -INFINITY;
     Kahan z;
     z.init();
+    // The half's exp2 sum is added to z only after the next half's exp2 terms
+    // are issued (its terms have arrived by then); adding it at once would
+    // stall the warp until the exp2 unit has worked through its queue.
+    float pend = 0.f;
     for (int i = wg; i < ntiles; i += 2) {
       if (!warp_wait(&sm.tm_full[wg], (i >> 1) & 1, abort)) break;
       tc_fence_after();
@@ -266,6 +270,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           const float c = ex2(m - xm);
           z.s *= c;
           z.c *= c;
+          pend *= c;
           m = xm;
         }
         if (m != -INFINITY) {
@@ -275,10 +280,12 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           float ps[8];
 #pragma unroll
           for (int p = 0; p < 8; ++p) ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
-          z.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
+          z.add(pend);
+          pend = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
         }
       }
     }
+    z.add(pend);
     // merge the two warpgroups' statistics of each row
     if (wg == 1) sm.half[warp & 3][lane] = make_float2(m, z.s);
     __syncwarp();
@@ -313,12 +320,12 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __restrict__ part,
                                  const float* __restrict__ lse_nat, float* __restrict__ nlse) {
   const Req rq = tb.req[blockIdx.y];
-  const int cw = rq.C * (int)kTile;
-  const int64_t per = (int64_t)sh.L * sh.Hkv * cw;
+  const int rows = rq.C * rq.cw;              // padded rows of one (layer, KV head)
+  const int64_t per = (int64_t)sh.L * sh.Hkv * rows;
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= per) return;
-  const int p = (int)(i % cw);
-  const int grp = (int)(i / cw);
+  const int p = (int)(i % rows);
+  const int grp = (int)(i / rows);
   const int l = grp / sh.Hkv, g = grp % sh.Hkv;
   float out = -INFINITY;                      // padding rows: exp2(x + -inf) = 0
   if (p < sh.G * rq.W) {
@@ -344,15 +351,59 @@ __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __res
 //
 // A pair owns a tile of 256 keys (128 per CTA, keys in TMEM lanes) and walks
 // all layers: per layer its K rows (each CTA its own 128 keys, double
-// buffered), then the layer's window rows in chunks of 256 (each CTA loads
-// 128 rows of the chunk).  One 2-SM MMA chain (M = 256 keys, N = 256 rows,
-// K = 128) leaves each key's 256 logits in its own CTA's tensor memory.
-// Every CTA also loads the chunk's 256 row normalisers into its own shared
-// memory (rows past the row set carry -inf and add 0).  Warpgroup wg takes
-// the chunks q with q % 2 == wg (TMEM slot wg), all 256 columns in two
-// halves.
+// buffered), then the layer's G*W window rows in C chunks of cw <= 256 rows
+// (G*W spread evenly, rounded up to 16, so a 448-row set is two chunks of
+// 224, not two of 256; CTA r uses rows r*cw/2 ... of the chunk from a
+// 128-row box).  One 2-SM MMA chain (M = 256 keys, N = cw rows, K = 128)
+// leaves each key's cw logits in its own CTA's tensor memory.  Every CTA
+// also loads the chunk's cw row normalisers into its own shared memory (rows
+// past the row set carry -inf and add 0).  Warpgroup wg takes the chunks q
+// with q % 2 == wg (TMEM slot wg), the cw columns in up to two halves of 128.
 
 constexpr uint32_t kChunkRows = 256;            // window rows per pass-2 chunk (both CTAs)
+
+// One pass-2 consumer step over NP groups of 16 TMEM columns (one key per
+// lane, one window row per column) starting at col0: load, optionally free
+// the slot (last load of the chunk), then sum exp2(x * s2 + nl[col]) over the
+// columns.  NP is a compile-time count so the loads and sums unroll fully.
+template <int NP>
+__device__ __forceinline__ float colsum_group(uint32_t col0, const float* nl_col, float s2, bool release,
+                                              uint32_t tm_empty0, int lane) {
+  float x[NP][16];
+  {
+    uint32_t vv[NP][16];
+#pragma unroll
+    for (int p = 0; p < NP; ++p) tmem_ld16(col0 + p * 16, vv[p]);
+    tmem_wait_only();
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+      reg_fence(vv[p]);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(vv[p][j]);
+    }
+  }
+  if (release) {
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(tm_empty0);   // slot copied out
+  }
+  const float4* nl = reinterpret_cast<const float4*>(nl_col);
+  float ps[8];
+#pragma unroll
+  for (int p = 0; p < 8; ++p) ps[p] = 0.f;
+#pragma unroll
+  for (int p = 0; p < NP; ++p) {
+    float2 nb[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 f = nl[p * 4 + j];
+      nb[2 * j] = make_float2(f.x, f.y);
+      nb[2 * j + 1] = make_float2(f.z, f.w);
+    }
+    ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
+  }
+  return ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+}
 constexpr int kQStagesPair = 4;                 // Q ring of pass 2 (per CTA: 32 KB + 1 KB a stage)
 
 struct P2Smem {
@@ -385,8 +436,8 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
   const Req rq = tb.req[r];
   const int u = unit - tb.unit0_tc2[r];
   const int g = u / rq.tiles, kt = u % rq.tiles;
-  const int C = rq.C;                          // 128-row chunks per layer (even)
-  const int C2 = C >> 1;                       // 256-row chunks per layer
+  const int C2 = rq.C;                         // chunks per layer
+  const int cw = rq.cw;                        // rows per chunk (multiple of 16, <= 256)
   const int L = sh.L;
 
   if (threadIdx.x == 0) {
@@ -432,17 +483,17 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
       tma_load_2d_pair(sm.k[ks][0], &tmK, 0, ky, k_full0);
       tma_load_2d_pair(sm.k[ks][1], &tmK, 64, ky, k_full0);
       ++k_issued;
-      const int qy0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + (int)rank * (int)kTile;
+      const int qy0 = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + (int)rank * (cw >> 1);
       for (int c = 0; c < C2; ++c) {
         const int q = l * C2 + c, qs = q % kQStagesPair;
         if (!mbar_wait(&sm.q_empty[qs], ((q / kQStagesPair) & 1) ^ 1, abort)) { ok = false; break; }
         if (rank == 0) mbar_arrive_expect_tx(&sm.q_full[qs], 2 * kTileBytes);
         const uint32_t q_full0 = map_to_rank(smem_u32(&sm.q_full[qs]), 0);
-        tma_load_2d_pair(sm.q[qs][0], &tmQ, 0, qy0 + c * (int)kChunkRows, q_full0);
-        tma_load_2d_pair(sm.q[qs][1], &tmQ, 64, qy0 + c * (int)kChunkRows, q_full0);
-        mbar_arrive_expect_tx(&sm.nl_full[qs], kChunkRows * 4);
-        bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C2 + c) * kChunkRows,
-                  kChunkRows * 4, &sm.nl_full[qs]);
+        tma_load_2d_pair(sm.q[qs][0], &tmQ, 0, qy0 + c * cw, q_full0);
+        tma_load_2d_pair(sm.q[qs][1], &tmQ, 64, qy0 + c * cw, q_full0);
+        mbar_arrive_expect_tx(&sm.nl_full[qs], (uint32_t)cw * 4);
+        bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C2 + c) * cw,
+                  (uint32_t)cw * 4, &sm.nl_full[qs]);
         ++q_issued;
       }
     }
@@ -456,8 +507,8 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
         drain_wait(&sm.q_full[i % kQStagesPair], (i / kQStagesPair) & 1);
     }
   } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
-    // ---- MMA issuer (even CTA): D[key][row] = K_tile . Q_chunk^T, 256 x 256
-    const uint32_t idesc = idesc_bf16_f32(2 * kTile, kChunkRows);
+    // ---- MMA issuer (even CTA): D[key][row] = K_tile . Q_chunk^T, 256 x cw
+    const uint32_t idesc = idesc_bf16_f32(2 * kTile, (uint32_t)cw);
     bool ok = true;
     for (int l = 0; ok && l < L; ++l) {
       const int ks = l & 1;
@@ -490,73 +541,101 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     const float s2 = sh.scale_log2;
     const int v = kt * (int)kPairKeys + (int)rank * (int)kTile + key;
     const bool per_layer = sh.rank_mode == VC_RANK_PER_LAYER;
-    const int nq = L * C2;
-    Kahan tot, lay;
+    const int nhalf = (cw + (int)kTile - 1) / (int)kTile;   // 1 or 2 halves of 128 columns
+    // The sum of a group of exp2 terms is ready only once the exp2 unit has
+    // worked through the warp's queue, which takes long after the last one
+    // is issued.  So nothing waits for a sum right after issuing it: the last
+    // half-sum of a chunk stays pending until the next chunk's first half is
+    // issued, and a layer is added to the total only after the next layer's
+    // chunk is issued.  Layer l accumulates into a[l & 1]; the additions keep
+    // their order (halves in order into the layer, layers in order into the
+    // total).
+    Kahan tot, a0, a1;
     tot.init();
-    lay.init();
-    for (int q = 0; q < nq; ++q) {
-      const int l = q / C2, c = q % C2;
-      if ((q & 1) == wg) {
-        const int qs = q % kQStagesPair;
-        const bool go = __all_sync(0xffffffffu, *abort == 0);
-        if (go && warp_wait(&sm.tm_full[wg], (q >> 1) & 1, abort) &&
-            warp_wait(&sm.nl_full[qs], (q / kQStagesPair) & 1, abort)) {
-          tc_fence_after();
-#pragma unroll 1
-          for (int hf = 0; hf < 2; ++hf) {
-            const uint32_t col0 = tbase + lane_off + (uint32_t)wg * kChunkRows + (uint32_t)hf * kTile;
-            float x[8][16];
-            {
-              uint32_t vv[8][16];
-#pragma unroll
-              for (int p = 0; p < 8; ++p) tmem_ld16(col0 + p * 16, vv[p]);
-              tmem_wait_only();
-#pragma unroll
-              for (int p = 0; p < 8; ++p) {
-                reg_fence(vv[p]);
-#pragma unroll
-                for (int j = 0; j < 16; ++j) x[p][j] = __uint_as_float(vv[p][j]);
-              }
-            }
-            if (hf == 1) {
-              tc_fence_before();
-              __syncwarp();
-              if (lane == 0) mbar_arrive_cluster(tm_empty0);   // slot copied out
-            }
-            const float4* nl = reinterpret_cast<const float4*>(sm.nlse[qs] + hf * (int)kTile);
-            float ps[8];
-#pragma unroll
-            for (int p = 0; p < 8; ++p) {
-              float2 nb[8];
-#pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                const float4 f = nl[p * 4 + j];
-                nb[2 * j] = make_float2(f.x, f.y);
-                nb[2 * j + 1] = make_float2(f.z, f.w);
-              }
-              ps[p] = exp2_sum16(x[p], make_float2(s2, s2), nb);
-            }
-            lay.add(((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.q_empty[qs]);   // this warp is done with the stage's normalisers
+    a0.init();
+    a1.init();
+    float pend = 0.f;                               // last half-sum of the latest chunk
+    int pend_l = -1;                                // its layer (-1: none)
+    auto add_to_layer = [&](int l, float x) {
+      if (l & 1) a1.add(x);
+      else a0.add(x);
+    };
+    auto flush = [&](int l) {                       // the pending half-sum, if it is layer l's
+      if (pend_l == l) {
+        add_to_layer(l, pend);
+        pend_l = -1;
       }
-      if (c == C2 - 1) {
-        if (per_layer) {
-          sm.red[wg][key] = lay.s;
-          __syncwarp();
-          named_sync(1, 2 * kTile);
-          if (wg == 0 && v < rq.n)
-            scores[rq.s_off + ((int64_t)l * sh.Hkv + g) * rq.n + v] = sm.red[0][key] + sm.red[1][key];
-          named_sync(1, 2 * kTile);
+    };
+    auto half_sum = [&](int qs, int hf) -> float {
+      const int np = min(8, (cw >> 4) - hf * 8);    // 16-column groups of this half
+      const uint32_t col0 = tbase + lane_off + (uint32_t)wg * kChunkRows + (uint32_t)hf * kTile;
+      const float* nl = sm.nlse[qs] + hf * (int)kTile;
+      const bool rel = hf == nhalf - 1;             // the slot is free after this load
+      switch (np) {
+        case 8: return colsum_group<8>(col0, nl, s2, rel, tm_empty0, lane);
+        case 7: return colsum_group<7>(col0, nl, s2, rel, tm_empty0, lane);
+        case 6: return colsum_group<6>(col0, nl, s2, rel, tm_empty0, lane);
+        case 5: return colsum_group<5>(col0, nl, s2, rel, tm_empty0, lane);
+        case 4: return colsum_group<4>(col0, nl, s2, rel, tm_empty0, lane);
+        case 3: return colsum_group<3>(col0, nl, s2, rel, tm_empty0, lane);
+        case 2: return colsum_group<2>(col0, nl, s2, rel, tm_empty0, lane);
+        default: return colsum_group<1>(col0, nl, s2, rel, tm_empty0, lane);
+      }
+    };
+    // one chunk q (layer l) of this warpgroup: wait for its logits and
+    // normalisers, issue its exp2 terms, release the normaliser stage
+    auto run_chunk = [&](int q, int l) {
+      const int qs = q % kQStagesPair;
+      const bool go = __all_sync(0xffffffffu, *abort == 0);
+      if (go && warp_wait(&sm.tm_full[wg], (q >> 1) & 1, abort) &&
+          warp_wait(&sm.nl_full[qs], (q / kQStagesPair) & 1, abort)) {
+        tc_fence_after();
+        const float h0 = half_sum(qs, 0);
+        if (pend_l >= 0) {                          // the previous chunk's last half
+          add_to_layer(pend_l, pend);
+          pend_l = -1;
+        }
+        if (nhalf == 2) {
+          const float h1 = half_sum(qs, 1);
+          add_to_layer(l, h0);
+          pend = h1;
         } else {
-          tot.add(lay.s);
+          pend = h0;
         }
-        lay.init();
+        pend_l = l;
       }
-    }
-    if (!per_layer) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.q_empty[qs]);   // this warp is done with the stage's normalisers
+    };
+    auto layer_total = [&](int l) -> float {         // layer l's sum, its accumulator reset
+      flush(l);
+      const float t = (l & 1) ? a1.s : a0.s;
+      if (l & 1) a1.init();
+      else a0.init();
+      return t;
+    };
+    if (per_layer) {
+      for (int l = 0; l < L; ++l) {
+        for (int c = 0; c < C2; ++c) {
+          const int q = l * C2 + c;
+          if ((q & 1) == wg) run_chunk(q, l);
+        }
+        sm.red[wg][key] = layer_total(l);
+        __syncwarp();
+        named_sync(1, 2 * kTile);
+        if (wg == 0 && v < rq.n)
+          scores[rq.s_off + ((int64_t)l * sh.Hkv + g) * rq.n + v] = sm.red[0][key] + sm.red[1][key];
+        named_sync(1, 2 * kTile);
+      }
+    } else {
+      for (int l = 0; l < L; ++l) {
+        for (int c = 0; c < C2; ++c) {
+          const int q = l * C2 + c;
+          if ((q & 1) == wg) run_chunk(q, l);
+        }
+        if (l > 0) tot.add(layer_total(l - 1));
+      }
+      tot.add(layer_total(L - 1));
       sm.red[wg][key] = tot.s;
       __syncwarp();
       named_sync(1, 2 * kTile);

@@ -20,11 +20,11 @@ struct Req {                 // one request of a batch
   int64_t s_off;             // float offset of its scores [Hkv][n] or [L][Hkv][n]
   int64_t out_row0;          // first output row (K_out/V_out/idx_out)
   int64_t drop_row0;         // first drop-list row
-  int64_t lsep_off;          // float offset of its chunk-padded row normalisers [L][Hkv][C*128]
+  int64_t lsep_off;          // float offset of its chunk-padded row normalisers [L][Hkv][C*cw]
   int64_t vs_row0;           // first row of its compacted survivors' values (tensor-core fusion)
   int32_t n, W, Nq, h;
-  int32_t C;                 // 128-row chunks of one (layer, KV head) row set, padded to
-                             // whole 256-row chunks: 2*ceil(G*W/256)
+  int32_t C;                 // column-sum chunks of one (layer, KV head) row set, ceil(G*W/256)
+  int32_t cw;                // rows per chunk: G*W spread over C chunks, rounded up to 16
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
   int32_t tiles;             // 256-key tiles, ceil(n/256)
   int32_t chunk0;            // first 1024-key sort chunk of its first ranking problem

@@ -174,7 +174,10 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
   FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
-  const int unit = (int)(blockIdx.x >> 1);
+  // units in reverse order: later layers have fewer kept and more dropped
+  // rows, so their units are the longest; starting them first leaves the
+  // short units of the first layers to fill the last wave
+  const int unit = (int)(gridDim.x >> 1) - 1 - (int)(blockIdx.x >> 1);
 
   const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
   const int r = rl / sh.L;

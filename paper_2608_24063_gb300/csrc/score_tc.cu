@@ -12,7 +12,9 @@
 //   merge  (lse_merge)       -lse2 = -(m + log2 z) over the splits (or minus
 //                            the caller's natural-log normaliser * log2 e),
 //                            written per (layer, KV head) padded with -inf to
-//                            whole 256-row chunks;
+//                            whole pass-2 chunks; with a single key split
+//                            pass 1 writes these values itself and the merge
+//                            is skipped;
 //   pass 2 (score_colsum_tc) CTA pairs, keys in TMEM lanes: each thread owns
 //                            one key and sums exp2(x*scale*log2e - lse2[row])
 //                            over all rows of all layers (compensated),
@@ -118,7 +120,7 @@ struct P1Smem {
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                    Shape sh, Tables tb, int S, float2* __restrict__ part) {
+                    Shape sh, Tables tb, int S, float2* __restrict__ part, float* __restrict__ nlse) {
   extern __shared__ uint8_t smem_raw[];
   P1Smem& sm = *reinterpret_cast<P1Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -299,8 +301,18 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
         if (o.x != -INFINITY) zz += o.y * ex2(o.x - mm);
       }
       const int rho = rbp * 256 + (int)rank * (int)kTile + lrow;
-      if (rho < rows)
-        part[(rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho) * S + s] = make_float2(mm, zz);
+      if (S > 1) {
+        if (rho < rows)
+          part[(rq.lse_off + ((int64_t)l * sh.Hq + g * sh.G) * rq.W + rho) * S + s] = make_float2(mm, zz);
+      } else if (rho < rq.C * rq.cw) {
+        // one key split: the merge's result directly, same arithmetic
+        float out = -INFINITY;                      // padding rows: exp2(x + -inf) = 0
+        if (rho < rows) {
+          const float z = mm != -INFINITY ? zz * exp2f(0.f) : 0.f;
+          out = -(mm + log2f(z));
+        }
+        nlse[rq.lsep_off + ((int64_t)l * sh.Hkv + g) * (rq.C * rq.cw) + rho] = out;
+      }
     }
   }
   __syncwarp();
@@ -725,11 +737,11 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
     e = cudaFuncSetAttribute(score_lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
     if (e != cudaSuccess) return e;
     ProfileScope ps("score_lse_tc", st);
-    score_lse_tc_kernel<<<2 * tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part);
+    score_lse_tc_kernel<<<2 * tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part, nlse_pad);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  {
+  if (lse_nat || tp.S > 1) {
     ProfileScope ps("lse_merge", st);
     lse_merge_kernel<<<dim3((unsigned)((tp.max_prows + 255) / 256), sh.n_req), 256, 0, st>>>(
         sh, tb, tp.S, part, lse_nat, nlse_pad);

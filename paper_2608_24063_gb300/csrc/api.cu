@@ -21,13 +21,6 @@ constexpr size_t kAlign = 256;
 // Kernel path: VC_PATH_AUTO uses the tcgen05 score kernels for bf16, d = 128.
 std::atomic<int> g_path{VC_PATH_AUTO};
 
-int sm_count() {
-  int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-    return 148;
-  return n;
-}
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 // Sequential carving of the caller workspace into 256-byte aligned regions.

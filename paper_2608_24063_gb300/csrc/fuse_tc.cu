@@ -253,7 +253,6 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     const uint32_t id_s = idesc_bf16_f32(2 * kTile, kDTile);
     const uint32_t id_o = idesc_bf16_f32_bmn(2 * kTile, kTile);
     bool ok = mbar_wait(&sm.vk_pair, 0, abort);
-    int jo = 0;                                   // O products issued
     for (int j = 0; ok && j <= nt; ++j) {
       if (j < nt) {
         // S(j) into buffer j % 2 (its previous user O(j-2) was issued before)
@@ -280,13 +279,11 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
                            (jp > 0 || kk > 0) ? 1u : 0u);
         mma_commit_pair(&sm.vd_empty[st], 3);
         mma_commit_pair(&sm.o_done, 3);
-        jo = j;
       }
     }
     // always committed (also after a give-up), so the epilogue's wait ends
     mma_commit_pair(&sm.mma_done, 3);
     drain_wait(&sm.mma_done, 0);
-    (void)jo;
   } else if (warp < 8) {
     // ---- softmax over the drop set and epilogue: one kept row per TMEM lane
     const int q4 = warp & 3;                          // lane quadrant

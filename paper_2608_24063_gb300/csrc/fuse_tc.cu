@@ -179,7 +179,7 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
   // short units of the first layers to fill the last wave
   const int unit = (int)(gridDim.x >> 1) - 1 - (int)(blockIdx.x >> 1);
 
-  const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
+  const int rl = upper_index_warp(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
   const int r = rl / sh.L;
   const Req rq = tb.req[r];
   const Layer ly = tb.layer[rl];

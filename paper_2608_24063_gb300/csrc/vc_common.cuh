@@ -76,6 +76,18 @@ __device__ __forceinline__ int upper_index(const Int* prefix, int count, Int key
   return lo;
 }
 
+// The same index found by a whole warp at once: it is the number of entries
+// <= key, minus one (prefix is non-decreasing and prefix[0] = 0 <= key), so
+// each lane counts a strided share and the warp sums the counts.  All loads
+// are independent, so the lookup costs one memory latency instead of one per
+// bisection step.  Every lane of the warp must call it; all get the result.
+template <typename Int>
+__device__ __forceinline__ int upper_index_warp(const Int* prefix, int count, Int key) {
+  int c = 0;
+  for (int i = (int)(threadIdx.x & 31); i < count; i += 32) c += prefix[i] <= key ? 1 : 0;
+  return __reduce_add_sync(0xffffffffu, c) - 1;
+}
+
 // ---------------------------------------------------------------------------
 // Element access.
 

@@ -1,0 +1,257 @@
+"""Planted mistakes in the oracle: every one must be caught by the pins.
+
+Each case replaces one oracle function (on the CPU, for this test only) with
+a copy that carries a single plausible mistake -- a dropped term, a wrong
+sign, index or axis, a transposed or swapped operand, an off-by-one -- and
+runs the pin tests of that part of the oracle (test_oracle_plan,
+test_oracle_scores, test_oracle_select_fuse).  At least one pin must fail.
+
+The pins used here check the oracle against things other than itself: values
+and closed forms from the paper, brute force on tiny inputs, invariants, and
+library routines (torch softmax / SDPA).  The stored golden budgets are left
+out on purpose: they were written by the oracle, so they would catch a change
+but prove nothing about correctness.
+"""
+import inspect
+import itertools
+from fractions import Fraction
+from math import floor
+
+import numpy as np
+import pytest
+
+from oracle import plan
+from oracle import prunekv as ok
+from tests import test_oracle_plan as pins_plan
+from tests import test_oracle_scores as pins_scores
+from tests import test_oracle_select_fuse as pins_select_fuse
+
+SELF_PINS = {"test_golden_budgets_match_oracle"}
+
+
+def _pin_calls(module):
+    """Every test function of a pin module with its parametrize grid expanded."""
+    for name, fn in inspect.getmembers(module, inspect.isfunction):
+        if not name.startswith("test_") or name in SELF_PINS or fn.__module__ != module.__name__:
+            continue
+        grids = []
+        for mark in getattr(fn, "pytestmark", []):
+            if mark.name != "parametrize":
+                continue
+            names = mark.args[0]
+            names = [s.strip() for s in names.split(",")] if isinstance(names, str) else list(names)
+            combos = []
+            for v in mark.args[1]:
+                v = v.values if hasattr(v, "values") else v
+                v = tuple(v) if len(names) > 1 else (v,)
+                combos.append(dict(zip(names, v)))
+            grids.append(combos)
+        for combo in itertools.product(*grids) if grids else [()]:
+            kw = {}
+            for part in combo:
+                kw.update(part)
+            yield name, fn, kw
+
+
+def _failing_pins(modules):
+    failed = []
+    for mod in modules:
+        for name, fn, kw in _pin_calls(mod):
+            try:
+                fn(**kw)
+            except Exception:      # an assertion, or a crash a real run would report
+                failed.append(name)
+    return sorted(set(failed))
+
+
+# ---------------------------------------------------------------------------
+# mutated copies of oracle functions (one planted mistake each)
+
+def _softmax_rows(x):
+    m = x.max(axis=-1, keepdims=True)
+    e = np.exp(x - m)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def _attention(Qw_l, K_l, scale, row_lse=None, kv=lambda j, G, Hkv: j // G, use_scale=True,
+               axis_rows=False, lse_sign=-1.0):
+    Hq, W, d = Qw_l.shape
+    Hkv = K_l.shape[0]
+    G = Hq // Hkv
+    out = np.empty((Hq, W, K_l.shape[1]))
+    for j in range(Hq):
+        x = Qw_l[j] @ K_l[kv(j, G, Hkv)].T
+        if use_scale:
+            x = x * scale
+        if row_lse is not None:
+            out[j] = np.exp(x + lse_sign * row_lse[j][:, None])
+        elif axis_rows:
+            out[j] = _softmax_rows(x.T).T
+        else:
+            out[j] = _softmax_rows(x)
+    return out
+
+
+def _scores(Qw, K, scale=None, rank_mode="shared", row_lse=None, mean=True, heads=None):
+    L, Hq, W, d = Qw.shape
+    _, Hkv, n, _ = K.shape
+    G = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / np.sqrt(d)
+    per_layer = np.zeros((L, Hkv, n))
+    for l in range(L):
+        A = ok.attention_weights(Qw[l], K[l], scale, None if row_lse is None else row_lse[l])
+        for g in range(Hkv):
+            hi = (g + 1) * G if heads is None else g * G + heads
+            per_layer[l, g] = A[g * G:hi].sum(axis=(0, 1))
+    if rank_mode == "per_layer":
+        return per_layer
+    return per_layer.sum(axis=0) / (L if mean else 1)
+
+
+def _select(s, B, Nq, rank_mode="shared", order_fn=None, drop_from=0, drop_to=0, sort_keep=True):
+    L = len(B)
+    Hkv = s.shape[-2]
+    keep = [[None] * Hkv for _ in range(L)]
+    drop = [[None] * Hkv for _ in range(L)]
+    rank = np.empty(s.shape, dtype=np.int64)
+    rank_fn = order_fn or ok.ranking
+    for g in range(Hkv):
+        for l in range(L):
+            sv = s[l, g] if rank_mode == "per_layer" else s[g]
+            order = rank_fn(sv)
+            if rank_mode == "per_layer":
+                rank[l, g, order] = np.arange(order.size)
+            elif l == 0:
+                rank[g, order] = np.arange(order.size)
+            kp = order[:B[l]]
+            keep[l][g] = (np.sort(kp) if sort_keep else kp) if B[l] > 0 else np.zeros(0, np.int64)
+            drop[l][g] = (np.sort(order[B[l] + drop_from:Nq + drop_to]) if B[l] > 0
+                          else np.zeros(0, np.int64))
+    return keep, drop, rank
+
+
+def _fuse(V_lg, keep_lg, drop_lg, mu, tau, phi_axis=-1, swap_mu=False, use_tau=True,
+          empty_zero=False):
+    Vk = V_lg[keep_lg]
+    if drop_lg.size == 0:
+        return np.zeros_like(Vk) if empty_zero else Vk.copy()
+    Vd = V_lg[drop_lg]
+    Z = Vk @ Vd.T
+    if use_tau:
+        Z = Z / tau
+    Phi = _softmax_rows(Z) if phi_axis == -1 else _softmax_rows(Z.T).T
+    a, b = (1.0 - mu, mu) if swap_mu else (mu, 1.0 - mu)
+    return a * Vk + b * (Phi @ Vd)
+
+
+def _parabolic_no_half(h):
+    if h == 1:
+        return [Fraction(1)]
+    return [1 - Fraction((l - 1) ** 2, (h - 1) ** 2) for l in range(1, h + 1)]
+
+
+def _normalised_to_h(h, m):
+    b = plan.parabolic_proportions(h)
+    s = sum(b)
+    return [x * h / s for x in b]
+
+
+def _apportion_ties_high(total, weights):
+    W = sum(weights)
+    quotas = [total * w / W for w in weights]
+    base = [floor(q) for q in quotas]
+    left = total - sum(base)
+    order = sorted(range(len(weights)), key=lambda i: (-(quotas[i] - base[i]), -i))
+    for i in order[:left]:
+        base[i] += 1
+    return base
+
+
+def _default_h_floor(L):
+    h = floor(Fraction(3 * L, 4))
+    return max(min(2, L), min(h, L))
+
+
+def _plan_nq_without_m(L, n, rr, h=None, m=Fraction(3, 4)):
+    if h is None or h == 0:
+        h = plan.default_h(L)
+    T = plan.round_half_up(rr * n * L)
+    B = plan.apportion(T, plan.normalised_proportions(h, m)) + [0] * (L - h)
+    if B[0] > n:
+        raise plan.Infeasible("infeasible")
+    Nq = min(n, max(plan.round_half_up(Fraction(T) / h), B[0]))
+    return B, Nq, h
+
+
+def _plan_total_floor(L, n, rr, h=None, m=Fraction(3, 4)):
+    if h is None or h == 0:
+        h = plan.default_h(L)
+    T = floor(rr * n * L)
+    B = plan.apportion(T, plan.normalised_proportions(h, m)) + [0] * (L - h)
+    if B[0] > n:
+        raise plan.Infeasible("infeasible")
+    Nq = min(n, max(plan.round_half_up(Fraction(T) / (h * m)), B[0]))
+    return B, Nq, h
+
+
+SCORES = [pins_scores, pins_select_fuse]
+SELECT_FUSE = [pins_select_fuse]
+PLAN = [pins_plan]
+
+MUTATIONS = [
+    # scores (Eq. token_score)
+    ("shared score without the 1/L mean", ok, "token_scores",
+     lambda *a, **k: _scores(*a, mean=False, **k), SCORES),
+    ("only the first query head of each group", ok, "token_scores",
+     lambda *a, **k: _scores(*a, heads=1, **k), SCORES),
+    ("GQA map j % Hkv instead of j // G", ok, "attention_weights",
+     lambda *a: _attention(*a, kv=lambda j, G, Hkv: j % Hkv), SCORES),
+    ("logit scale 1/sqrt(d) dropped", ok, "attention_weights",
+     lambda *a: _attention(*a, use_scale=False), SCORES),
+    ("softmax over the window rows instead of the keys", ok, "attention_weights",
+     lambda *a: _attention(*a, axis_rows=True), SCORES),
+    ("prefill normaliser added instead of subtracted", ok, "attention_weights",
+     lambda *a: _attention(*a, lse_sign=1.0), SCORES),
+    # ranking and selection (Algorithm 1 steps 1 and 3)
+    ("ties to the higher index", ok, "ranking",
+     lambda s: np.lexsort((-np.arange(s.shape[0]), -s)), SELECT_FUSE),
+    ("ascending instead of descending scores", ok, "ranking",
+     lambda s: np.lexsort((np.arange(s.shape[0]), s)), SELECT_FUSE),
+    ("drop set starts one rank late", ok, "select",
+     lambda *a, **k: _select(*a, drop_from=1, **k), SELECT_FUSE),
+    ("drop set runs one rank past the survivors", ok, "select",
+     lambda *a, **k: _select(*a, drop_to=1, **k), SELECT_FUSE),
+    ("keep lists in rank order instead of position order", ok, "select",
+     lambda *a, **k: _select(*a, sort_keep=False, **k), SELECT_FUSE),
+    ("key compaction in reverse order", ok, "compact_keys",
+     lambda K_lg, keep_lg: K_lg[keep_lg[::-1]], SELECT_FUSE),
+    # value fusion (Eq. redistribution, Eq. weight_fusion)
+    ("Phi normalised over the kept rows", ok, "fuse_values",
+     lambda *a: _fuse(*a, phi_axis=0), SELECT_FUSE),
+    ("mu and 1 - mu swapped", ok, "fuse_values",
+     lambda *a: _fuse(*a, swap_mu=True), SELECT_FUSE),
+    ("temperature ignored", ok, "fuse_values",
+     lambda *a: _fuse(*a, use_tau=False), SELECT_FUSE),
+    ("empty drop set gives zeros", ok, "fuse_values",
+     lambda *a: _fuse(*a, empty_zero=True), SELECT_FUSE),
+    # budgets (Eq. parabolic, its normalisation, Sec. 4 defaults)
+    ("parabola without the factor 2", plan, "parabolic_proportions", _parabolic_no_half, PLAN),
+    ("proportions normalised to h instead of h*m", plan, "normalised_proportions",
+     _normalised_to_h, PLAN),
+    ("largest-remainder ties to the higher layer", plan, "apportion", _apportion_ties_high, PLAN),
+    ("truncation layer floor(3L/4) instead of rounded", plan, "default_h", _default_h_floor, PLAN),
+    ("survivors T/h without m", plan, "plan_budgets", _plan_nq_without_m, PLAN),
+    ("total T rounded down", plan, "plan_budgets", _plan_total_floor, PLAN),
+]
+
+
+def test_pins_pass_on_the_oracle():
+    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse]) == []
+
+
+@pytest.mark.parametrize("what,module,attr,mutant,pins", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(monkeypatch, what, module, attr, mutant, pins):
+    monkeypatch.setattr(module, attr, mutant)
+    caught = _failing_pins(pins)
+    assert caught, "no pin fails with the mistake: %s" % what

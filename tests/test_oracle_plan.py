@@ -44,6 +44,12 @@ def test_default_truncation_from_paper():
     assert plan.default_h(1) == 1 and plan.default_h(2) == 2
 
 
+def test_truncation_rounds_half_up():
+    # The paper gives h = 3L/4 only where it is whole; the reading for other
+    # depths rounds half up (4.5 -> 5, 7.5 -> 8, 22.5 -> 23, 5.25 -> 5).
+    assert [plan.default_h(L) for L in (6, 10, 30, 7)] == [5, 8, 23, 5]
+
+
 def test_rr_product_example_from_paper():
     # Sec. 4: p=0.75, q=0.67, h=3L/4, m=0.75 give RR ~ 28%.
     p, q, m = Fraction(3, 4), Fraction(67, 100), Fraction(3, 4)

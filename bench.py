@@ -44,6 +44,10 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time direct launches instead of a CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
+                    help="layer-budget schedule (the paper's ablation axes); parabola is the method")
+    ap.add_argument("--drop", choices=["survivors", "all"], default="survivors",
+                    help="drop set: survivors of the top-q step (method) or every non-kept token")
     return ap.parse_args()
 
 
@@ -60,10 +64,15 @@ def peaks():
 # ---------------------------------------------------------------------------
 # Algorithmic work of one pass (what the method must do, each logit once).
 
-def plans_for(wl, vc):
+SCHEDULES = {"parabola": 0, "fixed": 1, "arithmetic": 2, "geometric": 3}
+DROPS = {"survivors": 0, "all": 1}
+
+
+def plans_for(wl, vc, schedule="parabola", drop="survivors"):
     out = []
     for r in wl.requests:
-        B, Nq, h = vc.viscache_plan_budgets(wl.L, r.n, r.rr_num, r.rr_den)
+        B, Nq, h = vc.viscache_plan_budgets_ex(wl.L, r.n, r.rr_num, r.rr_den, 0, 3, 4,
+                                               SCHEDULES[schedule], DROPS[drop])
         out.append((B, Nq, h))
     return out
 
@@ -172,7 +181,7 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------
-def oracle_sample(wl, layers, seed_layer0=0):
+def oracle_sample(wl, layers, seed_layer0=0, schedule="parabola", drop="survivors"):
     """Run the fp64 oracle on the first `layers` layers of request 0; returns (seconds, tokens*layers)."""
     import numpy as np
     import torch
@@ -187,7 +196,7 @@ def oracle_sample(wl, layers, seed_layer0=0):
     k, v = synth.make_kv(sub, 0, q)
     Qn, Kn, Vn = (t.to(torch.float64).numpy() for t in (q, k, v))
     r = sub.requests[0]
-    B, Nq, h = oplan.plan_budgets(layers, r.n, Fraction(r.rr_num, r.rr_den))
+    B, Nq, h = oplan.plan_budgets(layers, r.n, Fraction(r.rr_num, r.rr_den), schedule=schedule, drop=drop)
     t0 = time.perf_counter()
     ok.prunekv(Qn, Kn, Vn, B, Nq, mu=0.7, tau=1.0)
     dt = time.perf_counter() - t0
@@ -208,15 +217,15 @@ def run_reference(args, wl):
         return
     layers = 1
     for _ in range(args.warmup):
-        oracle_sample(wl, layers)
+        oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop)
     times = []
     tl = 0
     for _ in range(args.steps):
-        dt, tl = oracle_sample(wl, layers)
+        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop)
         times.append(dt)
     sec = sum(times) / len(times)
     val = tl / sec
-    cfg = workload_config(wl)
+    cfg = workload_config(wl, args)
     line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
@@ -251,7 +260,7 @@ def job_value(units_per_rank, world, ms_per_step):
     return world * units_per_rank / (ms_per_step * 1e-3)
 
 
-def workload_config(wl):
+def workload_config(wl, args=None):
     r = wl.requests[0]
     in_bytes = sum(wl.L * (wl.Hq * q.W + 2 * wl.Hkv * q.n) * wl.d * (2 if wl.dtype == "bf16" else 4)
                    for q in wl.requests)
@@ -260,6 +269,7 @@ def workload_config(wl):
             "W": [q.W for q in wl.requests],
             "retention": ["%d/%d" % (q.rr_num, q.rr_den) for q in wl.requests],
             "h": "3L/4", "m": 0.75, "mu": 0.7, "tau": 1.0, "rank": "shared",
+            "schedule": getattr(args, "schedule", "parabola"), "drop": getattr(args, "drop", "survivors"),
             "l2": "inputs larger than L2 (%.2f GB of Qw+K+V > 129 MB)" % (in_bytes / 1e9)}
 
 
@@ -293,7 +303,8 @@ def main():
     del qs, ks, vs
     batch = vc.Batch([r.n for r in wl.requests], [r.W for r in wl.requests],
                      [(r.rr_num, r.rr_den) for r in wl.requests])
-    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16 if wl.dtype == "bf16" else vc.VC_F32)
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16 if wl.dtype == "bf16" else vc.VC_F32,
+                         schedule=SCHEDULES[args.schedule], drop_mode=DROPS[args.drop])
     rows = vc.compressed_rows(batch, prm)
     K_out = torch.empty((rows, wl.d), dtype=K.dtype, device=dev)
     V_out = torch.empty((rows, wl.d), dtype=V.dtype, device=dev)
@@ -362,7 +373,7 @@ def main():
     vc.viscache_profile_enable(False)
     assert vc.prunekv_get_status(ws) == vc.VC_OK
 
-    plans = plans_for(wl, vc)
+    plans = plans_for(wl, vc, args.schedule, args.drop)
     work = algorithmic(wl, plans)
     value = job_value(work["tokens_layers"], world, ms_step)
     pk = peaks()
@@ -473,9 +484,9 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        dt1, tl1 = oracle_sample(wl, 1)
+        dt1, tl1 = oracle_sample(wl, 1, schedule=args.schedule, drop=args.drop)
         layers = max(1, min(wl.L, int(args.cpu_seconds / max(dt1, 1e-3))))
-        dt, tl = oracle_sample(wl, layers) if layers > 1 else (dt1, tl1)
+        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop) if layers > 1 else (dt1, tl1)
         cpu = {"value": tl / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": "Algorithm 1 (fp64 numpy) on the first %d of %d layers of the workload's "
                          "request (all %d tokens, %d window rows): %.1f s" %
@@ -488,7 +499,7 @@ def main():
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16"
                 if wl.dtype == "bf16" else "f32",
                 "data": "synthetic (seeded, structure of the paper's long-video workloads)",
-                "config": dict(workload_config(wl), launch="cuda graph of the prunekv_compress call"
+                "config": dict(workload_config(wl, args), launch="cuda graph of the prunekv_compress call"
                                if graph is not None else "direct prunekv_compress calls"),
                 "roofline": roof, "pass_roofline": pass_roof,
                 "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,

@@ -91,6 +91,42 @@ int viscache_plan_budgets(int32_t L, int32_t n_vis, uint32_t rr_num, uint32_t rr
                           int32_t h, uint32_t m_num, uint32_t m_den,
                           int32_t* B_out, int32_t* n_survive_out, int32_t* h_out);
 
+/* Layer-budget schedules (the ablation axes of the paper's Table "ablation"). */
+#define VC_SCHED_PARABOLA   0  /* Eq. (parabolic), the method's schedule (default) */
+#define VC_SCHED_FIXED      1  /* uniform budget per kept layer */
+#define VC_SCHED_ARITHMETIC 2  /* arithmetic progression (PyramidKV-style) */
+#define VC_SCHED_GEOMETRIC  3  /* geometric progression over four layer blocks (PDrop-style) */
+
+/* Drop set of each layer. */
+#define VC_DROP_SURVIVORS 0    /* survivors of the top-q step minus the keep set (default) */
+#define VC_DROP_ALL       1    /* every token not kept (n - B_l), i.e. Nq = n */
+
+/*
+ * viscache_plan_budgets_ex -- viscache_plan_budgets with a budget schedule
+ * and a drop-set choice.  The table names the schedules only ("uniform",
+ * "arithmetic progression", "geometric progression across four layer
+ * blocks"); the readings keep everything else of the method fixed (layers
+ * l > h evicted, T = round(RR*n*L), largest remainder, Nq = round(T/(h*m))
+ * clamped to [B_1, n]) and give b_l for l = 1..h as:
+ *   VC_SCHED_PARABOLA    1 - (l-1)^2 / (2 (h-1)^2)
+ *   VC_SCHED_FIXED       1
+ *   VC_SCHED_ARITHMETIC  1 - (l-1) / (2 (h-1))      (same end points 1 and 1/2)
+ *   VC_SCHED_GEOMETRIC   (1/2)^k for block k = 0..min(4,h)-1 of a split of
+ *                        layers 1..h into min(4, h) contiguous blocks whose
+ *                        sizes differ by at most one (larger blocks first)
+ * (b_l = 1 for every schedule when h = 1).  With VC_DROP_ALL the survivors
+ * are all n tokens (Nq = n), so each layer's drop set is every token it does
+ * not keep (the alternative reading of V_d's n - b_l rows in Sec. 3.2).
+ *   schedule    one of VC_SCHED_*
+ *   drop_mode   VC_DROP_SURVIVORS or VC_DROP_ALL
+ * Other arguments and errors as viscache_plan_budgets; B_out is
+ * non-increasing for every schedule.
+ */
+int viscache_plan_budgets_ex(int32_t L, int32_t n_vis, uint32_t rr_num, uint32_t rr_den,
+                             int32_t h, uint32_t m_num, uint32_t m_den, int32_t schedule,
+                             int32_t drop_mode, int32_t* B_out, int32_t* n_survive_out,
+                             int32_t* h_out);
+
 /*
  * prunekv_score -- token importance, Eq. (token_score) / Algorithm 1 step 1.
  *
@@ -216,6 +252,8 @@ typedef struct {
     float tau;                /* redistribution temperature, paper default 1.0 */
     float scale;              /* logit scale, 0 -> 1/sqrt(d) */
     int32_t rank_mode;        /* VC_RANK_SHARED or VC_RANK_PER_LAYER */
+    int32_t schedule;         /* VC_SCHED_* layer-budget schedule (0 = parabola) */
+    int32_t drop_mode;        /* VC_DROP_SURVIVORS or VC_DROP_ALL */
 } vc_params;
 
 size_t prunekv_workspace_size(const vc_batch* batch, const vc_params* p);

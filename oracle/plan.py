@@ -22,6 +22,22 @@ Readings where the paper is silent (each listed in the design doc):
 * h = round(3L/4) clamped to [min(2, L), L]; for h = 1 the single layer keeps
   proportion 1 (the formula is 0/0 there);
 * round() is round-half-up on exact rationals.
+
+Budget schedules of the ablation table (Sec. 4.3, Table "ablation": "uniform
+budget per layer", "arithmetic progression", "geometric progression across
+four layer blocks"); the table names them only, so each replaces b_l and
+keeps everything else (layers l > h evicted, the normalisation to h*m, T,
+largest remainder, Nq):
+
+* fixed: b_l = 1;
+* arithmetic: b_l = 1 - (l-1)/(2(h-1)), the parabola's end points 1 and 1/2;
+* geometric: layers 1..h in min(4, h) contiguous blocks, sizes differing by
+  at most one (larger blocks first), block k with b = (1/2)^k;
+* all of them b = [1] when h = 1.
+
+Drop set: "survivors" (default) drops the survivors minus the keep set;
+"all" drops every token not kept (the other reading of V_d's n - b_l rows in
+Sec. 3.2), i.e. Nq = n.
 """
 from __future__ import annotations
 
@@ -47,9 +63,32 @@ def parabolic_proportions(h: int) -> List[Fraction]:
     return [1 - Fraction((l - 1) ** 2, 2 * (h - 1) ** 2) for l in range(1, h + 1)]
 
 
-def normalised_proportions(h: int, m: Fraction) -> List[Fraction]:
+SCHEDULES = ("parabola", "fixed", "arithmetic", "geometric")
+
+
+def schedule_proportions(h: int, schedule: str = "parabola") -> List[Fraction]:
+    """b_l for l = 1..h under one of the budget schedules (see the module notes)."""
+    if schedule not in SCHEDULES:
+        raise ValueError("unknown schedule %r" % schedule)
+    if schedule == "parabola":
+        return parabolic_proportions(h)
+    if h == 1:
+        return [Fraction(1)]
+    if schedule == "fixed":
+        return [Fraction(1)] * h
+    if schedule == "arithmetic":
+        return [1 - Fraction(l - 1, 2 * (h - 1)) for l in range(1, h + 1)]
+    nb = min(4, h)
+    per, extra = divmod(h, nb)
+    b = []
+    for k in range(nb):
+        b += [Fraction(1, 2 ** k)] * (per + (1 if k < extra else 0))
+    return b
+
+
+def normalised_proportions(h: int, m: Fraction, schedule: str = "parabola") -> List[Fraction]:
     """b_l rescaled so that their sum is h*m (normalisation after Eq. parabolic)."""
-    b = parabolic_proportions(h)
+    b = schedule_proportions(h, schedule)
     s = sum(b)
     return [x * h * m / s for x in b]
 
@@ -71,11 +110,14 @@ class Infeasible(ValueError):
 
 
 def plan_budgets(L: int, n: int, rr: Fraction, h: Optional[int] = None,
-                 m: Fraction = Fraction(3, 4)) -> Tuple[List[int], int, int]:
+                 m: Fraction = Fraction(3, 4), schedule: str = "parabola",
+                 drop: str = "survivors") -> Tuple[List[int], int, int]:
     """Integer budgets B[0..L-1], survivors Nq and truncation layer h.
 
     Raises ``Infeasible`` when the largest layer budget would exceed n.
     """
+    if drop not in ("survivors", "all"):
+        raise ValueError("unknown drop set %r" % drop)
     if L < 1 or n < 1:
         raise ValueError("L and n must be >= 1")
     if not (0 < rr <= 1) or not (0 < m <= 1):
@@ -85,9 +127,11 @@ def plan_budgets(L: int, n: int, rr: Fraction, h: Optional[int] = None,
     if not 1 <= h <= L:
         raise ValueError("h must be in [1, L]")
     T = round_half_up(rr * n * L)
-    B = apportion(T, normalised_proportions(h, m)) + [0] * (L - h)
+    B = apportion(T, normalised_proportions(h, m, schedule)) + [0] * (L - h)
     if B[0] > n:
         raise Infeasible("retention %s cannot be met with h=%d, m=%s" % (rr, h, m))
     Nq = round_half_up(Fraction(T) / (h * m))
     Nq = min(n, max(Nq, B[0]))
+    if drop == "all":
+        Nq = n
     return B, Nq, h

@@ -368,6 +368,8 @@ int plan_batch(const vc_batch* b, const vc_params* p, std::vector<RequestPlan>* 
   if (p->rank_mode != VC_RANK_SHARED && p->rank_mode != VC_RANK_PER_LAYER) return VC_ERR_INVALID_ARG;
   if (!(p->mu >= 0.f && p->mu <= 1.f) || !(p->tau > 0.f) || !(p->scale >= 0.f))
     return VC_ERR_INVALID_ARG;
+  if (p->schedule < VC_SCHED_PARABOLA || p->schedule > VC_SCHED_GEOMETRIC) return VC_ERR_INVALID_ARG;
+  if (p->drop_mode != VC_DROP_SURVIVORS && p->drop_mode != VC_DROP_ALL) return VC_ERR_INVALID_ARG;
   plans->assign(b->n_req, RequestPlan{});
   for (int r = 0; r < b->n_req; ++r) {
     RequestPlan& q = (*plans)[r];
@@ -375,8 +377,9 @@ int plan_batch(const vc_batch* b, const vc_params* p, std::vector<RequestPlan>* 
     q.W = b->W[r];
     if (q.n < 1 || q.n > 65536 || q.W < 1) return VC_ERR_INVALID_ARG;
     q.B.assign(p->L, 0);
-    const int rc = viscache_plan_budgets(p->L, q.n, b->rr_num[r], b->rr_den[r], p->h, p->m_num,
-                                         p->m_den, q.B.data(), &q.Nq, &q.h);
+    const int rc = viscache_plan_budgets_ex(p->L, q.n, b->rr_num[r], b->rr_den[r], p->h, p->m_num,
+                                            p->m_den, p->schedule, p->drop_mode, q.B.data(), &q.Nq,
+                                            &q.h);
     if (rc != VC_OK) return rc;
   }
   return VC_OK;

@@ -26,13 +26,15 @@ VC_ERR_UNSUPPORTED = 6
 VC_ERR_DEVICE_INDEX = 7
 VC_BF16, VC_F32 = 0, 1
 VC_RANK_SHARED, VC_RANK_PER_LAYER = 0, 1
+VC_SCHED_PARABOLA, VC_SCHED_FIXED, VC_SCHED_ARITHMETIC, VC_SCHED_GEOMETRIC = 0, 1, 2, 3
+VC_DROP_SURVIVORS, VC_DROP_ALL = 0, 1
 VC_PATH_AUTO, VC_PATH_SIMT = 0, 1
 
 _ERR_NAMES = {1: "VC_ERR_INVALID_ARG", 2: "VC_ERR_INFEASIBLE", 3: "VC_ERR_WORKSPACE",
               4: "VC_ERR_CUDA", 5: "VC_ERR_DEVICE_TIMEOUT", 6: "VC_ERR_UNSUPPORTED",
               7: "VC_ERR_DEVICE_INDEX"}
 
-EXPORTED = ("viscache_plan_budgets", "prunekv_score_workspace_size", "prunekv_score",
+EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_workspace_size", "prunekv_score",
             "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
@@ -56,7 +58,8 @@ class vc_params(ctypes.Structure):
     _fields_ = [("L", ctypes.c_int32), ("Hq", ctypes.c_int32), ("Hkv", ctypes.c_int32),
                 ("d", ctypes.c_int32), ("dtype", ctypes.c_int32), ("h", ctypes.c_int32),
                 ("m_num", ctypes.c_uint32), ("m_den", ctypes.c_uint32), ("mu", ctypes.c_float),
-                ("tau", ctypes.c_float), ("scale", ctypes.c_float), ("rank_mode", ctypes.c_int32)]
+                ("tau", ctypes.c_float), ("scale", ctypes.c_float), ("rank_mode", ctypes.c_int32),
+                ("schedule", ctypes.c_int32), ("drop_mode", ctypes.c_int32)]
 
 
 _lib = None
@@ -72,6 +75,8 @@ def lib() -> ctypes.CDLL:
         vp, i32, u32, f32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint32, ctypes.c_float, ctypes.c_size_t
         pi32 = ctypes.POINTER(ctypes.c_int32)
         L.viscache_plan_budgets.argtypes = [i32, i32, u32, u32, i32, u32, u32, pi32, pi32, pi32]
+        L.viscache_plan_budgets_ex.argtypes = [i32, i32, u32, u32, i32, u32, u32, i32, i32, pi32, pi32,
+                                               pi32]
         L.prunekv_score_workspace_size.argtypes = [i32, i32, i32]
         L.prunekv_score_workspace_size.restype = sz
         L.prunekv_score.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp, vp,
@@ -156,6 +161,18 @@ def viscache_plan_budgets(L: int, n_vis: int, rr_num: int, rr_den: int, h: int =
     _check("viscache_plan_budgets",
            lib().viscache_plan_budgets(L, n_vis, rr_num, rr_den, h, m_num, m_den, B,
                                        ctypes.byref(nq), ctypes.byref(hh)))
+    return list(B), nq.value, hh.value
+
+
+def viscache_plan_budgets_ex(L: int, n_vis: int, rr_num: int, rr_den: int, h: int = 0,
+                             m_num: int = 3, m_den: int = 4, schedule: int = VC_SCHED_PARABOLA,
+                             drop_mode: int = VC_DROP_SURVIVORS) -> Tuple[List[int], int, int]:
+    """Host planner with a budget schedule and drop-set choice: returns (B[L], Nq, h)."""
+    B = (ctypes.c_int32 * L)()
+    nq, hh = ctypes.c_int32(), ctypes.c_int32()
+    _check("viscache_plan_budgets_ex",
+           lib().viscache_plan_budgets_ex(L, n_vis, rr_num, rr_den, h, m_num, m_den, schedule,
+                                          drop_mode, B, ctypes.byref(nq), ctypes.byref(hh)))
     return list(B), nq.value, hh.value
 
 
@@ -268,8 +285,10 @@ class Batch:
 
 def make_params(L: int, Hq: int, Hkv: int, d: int, dtype: int, h: int = 0, m=(3, 4),
                 mu: float = 0.7, tau: float = 1.0, scale: float = 0.0,
-                rank_mode: int = VC_RANK_SHARED) -> vc_params:
-    return vc_params(L, Hq, Hkv, d, dtype, h, m[0], m[1], mu, tau, scale, rank_mode)
+                rank_mode: int = VC_RANK_SHARED, schedule: int = VC_SCHED_PARABOLA,
+                drop_mode: int = VC_DROP_SURVIVORS) -> vc_params:
+    return vc_params(L, Hq, Hkv, d, dtype, h, m[0], m[1], mu, tau, scale, rank_mode, schedule,
+                     drop_mode)
 
 
 def prunekv_workspace_size(batch: Batch, params: vc_params) -> int:
@@ -279,7 +298,8 @@ def prunekv_workspace_size(batch: Batch, params: vc_params) -> int:
 def compressed_rows(batch: Batch, params: vc_params) -> int:
     rows = 0
     for n, (a, b) in zip(batch.n_vis, batch.rr):
-        B, _, _ = viscache_plan_budgets(params.L, n, a, b, params.h, params.m_num, params.m_den)
+        B, _, _ = viscache_plan_budgets_ex(params.L, n, a, b, params.h, params.m_num, params.m_den,
+                                           params.schedule, params.drop_mode)
         rows += params.Hkv * sum(B)
     return rows
 

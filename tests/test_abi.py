@@ -51,6 +51,34 @@ def test_planner_matches_oracle_exhaustive_L(rr):
             assert got == (ref[0], ref[1], ref[2]), (L, n, rr)
 
 
+SCHED = [(vc.VC_SCHED_PARABOLA, "parabola"), (vc.VC_SCHED_FIXED, "fixed"),
+         (vc.VC_SCHED_ARITHMETIC, "arithmetic"), (vc.VC_SCHED_GEOMETRIC, "geometric")]
+
+
+@pytest.mark.parametrize("code,name", SCHED)
+@pytest.mark.parametrize("drop_code,drop", [(vc.VC_DROP_SURVIVORS, "survivors"), (vc.VC_DROP_ALL, "all")])
+def test_schedule_planner_matches_oracle(code, name, drop_code, drop):
+    for L in list(range(1, 41)) + [64, 80, 128]:
+        for n in (1, 7, 1000, 12544):
+            for rr in ((19, 100), (28, 100), (1, 3)):
+                try:
+                    ref = plan.plan_budgets(L, n, Fraction(*rr), schedule=name, drop=drop)
+                except plan.Infeasible:
+                    with pytest.raises(vc.VisCacheError) as ei:
+                        vc.viscache_plan_budgets_ex(L, n, *rr, 0, 3, 4, code, drop_code)
+                    assert ei.value.code == vc.VC_ERR_INFEASIBLE
+                    continue
+                got = vc.viscache_plan_budgets_ex(L, n, *rr, 0, 3, 4, code, drop_code)
+                assert got == (ref[0], ref[1], ref[2]), (L, n, rr, name, drop)
+
+
+def test_schedule_planner_rejects_unknown_choices():
+    for sched, drop in [(-1, 0), (4, 0), (0, 2), (0, -1)]:
+        with pytest.raises(vc.VisCacheError) as ei:
+            vc.viscache_plan_budgets_ex(28, 1000, 1, 5, 0, 3, 4, sched, drop)
+        assert ei.value.code == vc.VC_ERR_INVALID_ARG
+
+
 def test_planner_explicit_h_and_m():
     for L, h, m in [(28, 14, (1, 2)), (80, 80, (1, 1)), (5, 1, (3, 4)), (64, 48, (3, 4))]:
         ref = plan.plan_budgets(L, 5000, Fraction(1, 5), h=h, m=Fraction(*m))

@@ -313,3 +313,30 @@ def test_select_matches_oracle_ranking(n, mode):
             assert np.array_equal(drop[Hkv * Qd + g * D:Hkv * Qd + (g + 1) * D], drop_ref[l][g])
         P += B[l]
         Qd += D
+
+
+SCHEDULES = [(vc.VC_SCHED_PARABOLA, "parabola"), (vc.VC_SCHED_FIXED, "fixed"),
+             (vc.VC_SCHED_ARITHMETIC, "arithmetic"), (vc.VC_SCHED_GEOMETRIC, "geometric")]
+
+
+@pytest.mark.parametrize("drop_code,drop", [(vc.VC_DROP_SURVIVORS, "survivors"), (vc.VC_DROP_ALL, "all")],
+                         ids=["survivors", "drop_all"])
+@pytest.mark.parametrize("code,name", SCHEDULES, ids=[s for _, s in SCHEDULES])
+def test_budget_schedules_match_oracle(code, name, drop_code, drop, kernel_path):
+    """The ablation schedules and the drop-all reading: same kernels, other plans."""
+    from fractions import Fraction
+    L, Hq, Hkv, d, n, W, rr = 6, 8, 2, 128, 1000, 16, (28, 100)
+    Q, K, V = (_rand(s, 900 + i, torch.bfloat16) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)], 1))
+    B, Nq, h = vc.viscache_plan_budgets_ex(L, n, *rr, 0, 3, 4, code, drop_code)
+    assert (B, Nq, h) == oplan.plan_budgets(L, n, Fraction(*rr), schedule=name, drop=drop)
+    out = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq)
+    log = check_request(Q, K, V, B, Nq, out, 0.7, 1.0)
+    assert len(log) <= 2, log
+    # the fused entry point with the same plan choices
+    batch = vc.Batch([n], [W], [rr])
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16, schedule=code, drop_mode=drop_code)
+    Ko, Vo, idx = vc.prunekv_compress(batch, prm, Q.to(DEV), K.to(DEV), V.to(DEV))
+    torch.cuda.synchronize()
+    assert torch.equal(idx, out["keep"]) and torch.equal(Ko, out["K_out"])
+    assert torch.equal(Vo, out["V_out"])

@@ -151,8 +151,8 @@ def _parabolic_no_half(h):
     return [1 - Fraction((l - 1) ** 2, (h - 1) ** 2) for l in range(1, h + 1)]
 
 
-def _normalised_to_h(h, m):
-    b = plan.parabolic_proportions(h)
+def _normalised_to_h(h, m, schedule="parabola"):
+    b = plan.schedule_proportions(h, schedule)
     s = sum(b)
     return [x * h / s for x in b]
 
@@ -168,31 +168,59 @@ def _apportion_ties_high(total, weights):
     return base
 
 
+def _schedule_mutant(arith_end=Fraction(1, 2), geo_ratio=Fraction(1, 2), small_blocks_first=False):
+    def fn(h, schedule="parabola"):
+        if schedule == "arithmetic" and h > 1:
+            return [1 - (1 - arith_end) * Fraction(l - 1, h - 1) for l in range(1, h + 1)]
+        if schedule == "geometric" and h > 1:
+            nb = min(4, h)
+            per, extra = divmod(h, nb)
+            sizes = [per + (1 if k < extra else 0) for k in range(nb)]
+            if small_blocks_first:
+                sizes = sizes[::-1]
+            b = []
+            for k in range(nb):
+                b += [geo_ratio ** k] * sizes[k]
+            return b
+        return _ORIG_SCHEDULE(h, schedule)
+    return fn
+
+
+_ORIG_SCHEDULE = plan.schedule_proportions
+
+
+def _plan_drop_all_ignored(L, n, rr, h=None, m=Fraction(3, 4), schedule="parabola", drop="survivors"):
+    return _ORIG_PLAN(L, n, rr, h, m, schedule)
+
+
+_ORIG_PLAN = plan.plan_budgets
+
+
 def _default_h_floor(L):
     h = floor(Fraction(3 * L, 4))
     return max(min(2, L), min(h, L))
 
 
-def _plan_nq_without_m(L, n, rr, h=None, m=Fraction(3, 4)):
+def _plan_nq_without_m(L, n, rr, h=None, m=Fraction(3, 4), schedule="parabola", drop="survivors"):
     if h is None or h == 0:
         h = plan.default_h(L)
     T = plan.round_half_up(rr * n * L)
-    B = plan.apportion(T, plan.normalised_proportions(h, m)) + [0] * (L - h)
+    B = plan.apportion(T, plan.normalised_proportions(h, m, schedule)) + [0] * (L - h)
     if B[0] > n:
         raise plan.Infeasible("infeasible")
     Nq = min(n, max(plan.round_half_up(Fraction(T) / h), B[0]))
-    return B, Nq, h
+    return B, (n if drop == "all" else Nq), h
 
 
-def _plan_total_floor(L, n, rr, h=None, m=Fraction(3, 4)):
+def _plan_total_floor(L, n, rr, h=None, m=Fraction(3, 4), schedule="parabola", drop="survivors"):
     if h is None or h == 0:
         h = plan.default_h(L)
     T = floor(rr * n * L)
-    B = plan.apportion(T, plan.normalised_proportions(h, m)) + [0] * (L - h)
+    B = plan.apportion(T, plan.normalised_proportions(h, m, schedule)) + [0] * (L - h)
     if B[0] > n:
         raise plan.Infeasible("infeasible")
     Nq = min(n, max(plan.round_half_up(Fraction(T) / (h * m)), B[0]))
-    return B, Nq, h
+    return B, (n if drop == "all" else Nq), h
 
 
 SCORES = [pins_scores, pins_select_fuse]
@@ -243,6 +271,13 @@ MUTATIONS = [
     ("truncation layer floor(3L/4) instead of rounded", plan, "default_h", _default_h_floor, PLAN),
     ("survivors T/h without m", plan, "plan_budgets", _plan_nq_without_m, PLAN),
     ("total T rounded down", plan, "plan_budgets", _plan_total_floor, PLAN),
+    ("arithmetic schedule ending at 1/3", plan, "schedule_proportions",
+     _schedule_mutant(arith_end=Fraction(1, 3)), PLAN),
+    ("geometric ratio 2/3 per block", plan, "schedule_proportions",
+     _schedule_mutant(geo_ratio=Fraction(2, 3)), PLAN),
+    ("geometric blocks smaller first", plan, "schedule_proportions",
+     _schedule_mutant(small_blocks_first=True), PLAN),
+    ("drop-all reading ignored", plan, "plan_budgets", _plan_drop_all_ignored, PLAN),
 ]
 
 

@@ -112,3 +112,65 @@ def test_golden_budgets_match_oracle():
     for case in gold["cases"]:
         B, Nq, h = plan.plan_budgets(case["L"], case["n"], Fraction(case["rr_num"], case["rr_den"]))
         assert (B, Nq, h) == (case["B"], case["Nq"], case["h"])
+
+
+# ---------------------------------------------------------------------------
+# budget schedules of the ablation table (readings in oracle/plan.py)
+
+SCHED_CASES = [(28, 12544, Fraction(19, 100)), (28, 3136, Fraction(28, 100)),
+               (80, 32768, Fraction(22, 100)), (5, 97, Fraction(1, 3)), (6, 1000, Fraction(1, 4)),
+               (3, 50, Fraction(2, 5))]
+
+
+@pytest.mark.parametrize("schedule", plan.SCHEDULES)
+@pytest.mark.parametrize("L,n,rr", SCHED_CASES)
+def test_schedule_closed_forms(schedule, L, n, rr):
+    B, Nq, h = plan.plan_budgets(L, n, rr, schedule=schedule)
+    T = floor(rr * n * L + Fraction(1, 2))
+    assert sum(B) == T                                   # same total for every schedule
+    assert all(b == 0 for b in B[h:])                    # layers l > h evicted
+    assert all(B[i] >= B[i + 1] for i in range(L - 1))   # non-increasing
+    assert min(n, max(B[0], floor(Fraction(T) / (h * Fraction(3, 4)) + Fraction(1, 2)))) == Nq
+
+
+def test_fixed_schedule_is_uniform():
+    # equal quotas: T // h each, the remainder to the lowest layers
+    for L, n, rr in SCHED_CASES:
+        B, _, h = plan.plan_budgets(L, n, rr, schedule="fixed")
+        T = sum(B)
+        assert B[:h] == [T // h + (1 if l < T % h else 0) for l in range(h)]
+
+
+def test_arithmetic_schedule_is_linear_from_one_to_half():
+    for h in (2, 3, 7, 21, 60):
+        b = plan.schedule_proportions(h, "arithmetic")
+        assert b[0] == 1 and b[-1] == Fraction(1, 2)
+        steps = {b[i] - b[i + 1] for i in range(h - 1)}
+        assert steps == {Fraction(1, 2 * (h - 1))}
+    B, _, h = plan.plan_budgets(28, 12544, Fraction(19, 100), schedule="arithmetic")
+    diffs = [B[i] - B[i + 1] for i in range(h - 1)]
+    assert max(diffs) - min(diffs) <= 2                  # integer budgets still linear
+
+
+def test_geometric_schedule_blocks():
+    for h in (1, 2, 3, 4, 5, 21, 60):
+        b = plan.schedule_proportions(h, "geometric")
+        assert len(b) == h
+        runs = [len(list(g)) for _, g in itertools.groupby(b)]
+        assert len(runs) == min(4, h)                                  # four blocks (fewer if h < 4)
+        assert max(runs) - min(runs) <= 1 and runs == sorted(runs, reverse=True)
+        levels = [k for k, _ in itertools.groupby(b)]
+        assert levels[0] == 1 and all(levels[i + 1] * 2 == levels[i] for i in range(len(levels) - 1))
+
+
+def test_schedules_coincide_for_one_layer():
+    for schedule in plan.SCHEDULES:
+        assert plan.plan_budgets(1, 1024, Fraction(1, 4), schedule=schedule) == ([256], 341, 1)
+
+
+def test_drop_all_keeps_budgets_and_takes_every_token():
+    for L, n, rr in SCHED_CASES:
+        for schedule in plan.SCHEDULES:
+            B, Nq, h = plan.plan_budgets(L, n, rr, schedule=schedule)
+            B2, Nq2, h2 = plan.plan_budgets(L, n, rr, schedule=schedule, drop="all")
+            assert (B2, h2) == (B, h) and Nq2 == n

@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
                     help="layer-budget schedule (the paper's ablation axes); parabola is the method")
+    ap.add_argument("--rank", choices=["shared", "per_layer"], default="shared",
+                    help="ranking: one order per KV head from the layer mean (method default) or per layer")
     ap.add_argument("--drop", choices=["survivors", "all"], default="survivors",
                     help="drop set: survivors of the top-q step (method) or every non-kept token")
     return ap.parse_args()
@@ -181,7 +183,7 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------
-def oracle_sample(wl, layers, seed_layer0=0, schedule="parabola", drop="survivors"):
+def oracle_sample(wl, layers, seed_layer0=0, schedule="parabola", drop="survivors", rank="shared"):
     """Run the fp64 oracle on the first `layers` layers of request 0; returns (seconds, tokens*layers)."""
     import numpy as np
     import torch
@@ -198,7 +200,7 @@ def oracle_sample(wl, layers, seed_layer0=0, schedule="parabola", drop="survivor
     r = sub.requests[0]
     B, Nq, h = oplan.plan_budgets(layers, r.n, Fraction(r.rr_num, r.rr_den), schedule=schedule, drop=drop)
     t0 = time.perf_counter()
-    ok.prunekv(Qn, Kn, Vn, B, Nq, mu=0.7, tau=1.0)
+    ok.prunekv(Qn, Kn, Vn, B, Nq, mu=0.7, tau=1.0, rank_mode=rank)
     dt = time.perf_counter() - t0
     return dt, r.n * layers
 
@@ -217,11 +219,11 @@ def run_reference(args, wl):
         return
     layers = 1
     for _ in range(args.warmup):
-        oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop)
+        oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop, rank=args.rank)
     times = []
     tl = 0
     for _ in range(args.steps):
-        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop)
+        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop, rank=args.rank)
         times.append(dt)
     sec = sum(times) / len(times)
     val = tl / sec
@@ -268,7 +270,7 @@ def workload_config(wl, args=None):
             "Hkv": wl.Hkv, "d": wl.d, "n_vis": [q.n for q in wl.requests],
             "W": [q.W for q in wl.requests],
             "retention": ["%d/%d" % (q.rr_num, q.rr_den) for q in wl.requests],
-            "h": "3L/4", "m": 0.75, "mu": 0.7, "tau": 1.0, "rank": "shared",
+            "h": "3L/4", "m": 0.75, "mu": 0.7, "tau": 1.0, "rank": getattr(args, "rank", "shared"),
             "schedule": getattr(args, "schedule", "parabola"), "drop": getattr(args, "drop", "survivors"),
             "l2": "inputs larger than L2 (%.2f GB of Qw+K+V > 129 MB)" % (in_bytes / 1e9)}
 
@@ -304,7 +306,8 @@ def main():
     batch = vc.Batch([r.n for r in wl.requests], [r.W for r in wl.requests],
                      [(r.rr_num, r.rr_den) for r in wl.requests])
     prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16 if wl.dtype == "bf16" else vc.VC_F32,
-                         schedule=SCHEDULES[args.schedule], drop_mode=DROPS[args.drop])
+                         schedule=SCHEDULES[args.schedule], drop_mode=DROPS[args.drop],
+                         rank_mode=vc.VC_RANK_PER_LAYER if args.rank == "per_layer" else vc.VC_RANK_SHARED)
     rows = vc.compressed_rows(batch, prm)
     K_out = torch.empty((rows, wl.d), dtype=K.dtype, device=dev)
     V_out = torch.empty((rows, wl.d), dtype=V.dtype, device=dev)
@@ -484,9 +487,9 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        dt1, tl1 = oracle_sample(wl, 1, schedule=args.schedule, drop=args.drop)
+        dt1, tl1 = oracle_sample(wl, 1, schedule=args.schedule, drop=args.drop, rank=args.rank)
         layers = max(1, min(wl.L, int(args.cpu_seconds / max(dt1, 1e-3))))
-        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop) if layers > 1 else (dt1, tl1)
+        dt, tl = oracle_sample(wl, layers, schedule=args.schedule, drop=args.drop, rank=args.rank) if layers > 1 else (dt1, tl1)
         cpu = {"value": tl / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": "Algorithm 1 (fp64 numpy) on the first %d of %d layers of the workload's "
                          "request (all %d tokens, %d window rows): %.1f s" %

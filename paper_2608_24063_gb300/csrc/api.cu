@@ -43,6 +43,7 @@ struct Layout {
   // inputs
   int n_req = 0, L = 0, Hq = 0, Hkv = 0, d = 0, rank_mode = VC_RANK_SHARED;
   bool need_lse = false, need_scores = false, need_sort = false, need_drop = false, need_vs = false;
+  bool prune_layers = false;   // score and rank only the layers the budgets keep (fused pass)
   // tensor-core score plan
   int S = 1;
   int64_t q_rows = 0, k_rows = 0, max_rows = 0, prows = 0, max_prows = 0;
@@ -115,8 +116,16 @@ struct Layout {
       max_prows = std::max<int64_t>(max_prows, (int64_t)L * Hkv * q.C * q.cw);
       q.nrb = (G * p.W + 255) / 256;
       q.tiles = (p.n + 255) / 256;
-      base_tc1[r] = L * Hkv * q.nrb;
-      u_tc2[r + 1] = u_tc2[r] + Hkv * q.tiles;
+      // per-layer ranking needs no scores of evicted layers (B_l = 0: a suffix,
+      // budgets are non-increasing); the shared ranking averages all layers
+      q.Ls = L;
+      if (prune_layers && rank_mode == VC_RANK_PER_LAYER && !p.B.empty()) {
+        q.Ls = 0;
+        for (int l = 0; l < L; ++l)
+          if (p.B[l] > 0) q.Ls = l + 1;
+      }
+      base_tc1[r] = q.Ls * Hkv * q.nrb;
+      u_tc2[r + 1] = u_tc2[r] + (q.Ls > 0 ? Hkv * q.tiles : 0);
       q_rows += (int64_t)L * Hq * p.W;
       k_rows += (int64_t)L * Hkv * p.n;
       max_rows = std::max<int64_t>(max_rows, (int64_t)L * Hq * p.W);
@@ -390,6 +399,7 @@ Layout compress_layout(const vc_params* p, const std::vector<RequestPlan>& plans
   lay.L = p->L; lay.Hq = p->Hq; lay.Hkv = p->Hkv; lay.d = p->d; lay.rank_mode = p->rank_mode;
   lay.need_lse = lay.need_scores = lay.need_sort = lay.need_drop = true;
   lay.need_vs = p->dtype == VC_BF16 && p->d == 128;
+  lay.prune_layers = true;
   lay.build(plans);
   return lay;
 }

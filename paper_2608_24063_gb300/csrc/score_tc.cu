@@ -451,6 +451,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
   const int C2 = rq.C;                         // chunks per layer
   const int cw = rq.cw;                        // rows per chunk (multiple of 16, <= 256)
   const int L = sh.L;
+  const int Ls = rq.Ls;                        // layers scored (all L unless per-layer ranking prunes)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
@@ -485,7 +486,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     prefetch_tmap(&tmK);
     int k_issued = 0, q_issued = 0;
     bool ok = true;
-    for (int l = 0; ok && l < L; ++l) {
+    for (int l = 0; ok && l < Ls; ++l) {
       const int ks = l & 1;
       if (!mbar_wait(&sm.k_empty[ks], ((l >> 1) & 1) ^ 1, abort)) break;
       if (rank == 0) mbar_arrive_expect_tx(&sm.k_full[ks], 2 * kTileBytes);
@@ -522,7 +523,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     // ---- MMA issuer (even CTA): D[key][row] = K_tile . Q_chunk^T, 256 x cw
     const uint32_t idesc = idesc_bf16_f32(2 * kTile, (uint32_t)cw);
     bool ok = true;
-    for (int l = 0; ok && l < L; ++l) {
+    for (int l = 0; ok && l < Ls; ++l) {
       const int ks = l & 1;
       if (!mbar_wait(&sm.k_full[ks], (l >> 1) & 1, abort)) break;
       for (int c = 0; c < C2; ++c) {
@@ -627,7 +628,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
       return t;
     };
     if (per_layer) {
-      for (int l = 0; l < L; ++l) {
+      for (int l = 0; l < Ls; ++l) {
         for (int c = 0; c < C2; ++c) {
           const int q = l * C2 + c;
           if ((q & 1) == wg) run_chunk(q, l);
@@ -640,14 +641,15 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
         named_sync(1, 2 * kTile);
       }
     } else {
-      for (int l = 0; l < L; ++l) {
+      // (Ls == L here: the shared ranking averages every layer)
+      for (int l = 0; l < Ls; ++l) {
         for (int c = 0; c < C2; ++c) {
           const int q = l * C2 + c;
           if ((q & 1) == wg) run_chunk(q, l);
         }
         if (l > 0) tot.add(layer_total(l - 1));
       }
-      tot.add(layer_total(L - 1));
+      if (Ls > 0) tot.add(layer_total(Ls - 1));
       sm.red[wg][key] = tot.s;
       __syncwarp();
       named_sync(1, 2 * kTile);

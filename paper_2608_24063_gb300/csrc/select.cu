@@ -40,14 +40,19 @@ __device__ __forceinline__ uint32_t desc_key(float s) {
 // element's rank is its position in its own chunk plus those counts: the
 // number of elements of the whole problem below it.
 
-__device__ __forceinline__ void problem_of(const Shape& sh, const Tables& tb, int p, Req& rq,
+// Ranking problem p: its request, score offset and chunk base; false when
+// the problem's layer is not scored (per-layer ranking of an evicted layer in
+// the fused pass), so the CTA has nothing to do.
+__device__ __forceinline__ bool problem_of(const Shape& sh, const Tables& tb, int p, Req& rq,
                                            int64_t& off, int64_t& chunk_base, int& nchunks) {
-  const int per_req = sh.rank_mode == VC_RANK_PER_LAYER ? sh.L * sh.Hkv : sh.Hkv;
+  const bool per_layer = sh.rank_mode == VC_RANK_PER_LAYER;
+  const int per_req = per_layer ? sh.L * sh.Hkv : sh.Hkv;
   const int r = p / per_req, k = p % per_req;
   rq = tb.req[r];
   nchunks = (rq.n + kSortChunk - 1) / kSortChunk;
   off = rq.s_off + (int64_t)k * rq.n;
   chunk_base = ((int64_t)rq.chunk0 + (int64_t)k * nchunks) * kSortChunk;
+  return !per_layer || k / sh.Hkv < rq.Ls;
 }
 
 // Compare-exchange of the bitonic network between lanes t and t ^ j of a
@@ -66,9 +71,9 @@ __global__ void __launch_bounds__(kSortChunk) chunk_sort_kernel(Shape sh, Tables
   Req rq;
   int64_t off, base;
   int nchunks;
-  problem_of(sh, tb, blockIdx.y, rq, off, base, nchunks);
+  const bool scored = problem_of(sh, tb, blockIdx.y, rq, off, base, nchunks);
   const int c = blockIdx.x;
-  if (c >= nchunks) return;
+  if (c >= nchunks || !scored) return;
   const int t = threadIdx.x;
   const int v = c * kSortChunk + t;
   uint64_t a = v < rq.n ? ((uint64_t)desc_key(scores[off + v]) << 32) | (uint32_t)v : ~0ull;
@@ -103,9 +108,9 @@ __global__ void __launch_bounds__(kSortChunk) chunk_rank_kernel(Shape sh, Tables
   Req rq;
   int64_t off, base;
   int nchunks;
-  problem_of(sh, tb, blockIdx.y, rq, off, base, nchunks);
+  const bool scored = problem_of(sh, tb, blockIdx.y, rq, off, base, nchunks);
   const int c = blockIdx.x;
-  if (c >= nchunks) return;
+  if (c >= nchunks || !scored) return;
   const int t = threadIdx.x;
   const uint64_t mine = chunks[base + (int64_t)c * kSortChunk + t];
   int count = t;                                   // elements of its own chunk below it

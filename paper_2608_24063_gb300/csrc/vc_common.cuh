@@ -28,6 +28,8 @@ struct Req {                 // one request of a batch
   int32_t nrb;               // 256-row blocks of that row set, ceil(G*W/256)
   int32_t tiles;             // 256-key tiles, ceil(n/256)
   int32_t chunk0;            // first 1024-key sort chunk of its first ranking problem
+  int32_t Ls;                // layers whose scores are needed: L, or in the fused pass with
+                             // per-layer ranking the leading layers with B_l > 0
 };
 
 struct Layer {               // one (request, layer)

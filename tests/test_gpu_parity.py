@@ -340,3 +340,20 @@ def test_budget_schedules_match_oracle(code, name, drop_code, drop, kernel_path)
     torch.cuda.synchronize()
     assert torch.equal(idx, out["keep"]) and torch.equal(Ko, out["K_out"])
     assert torch.equal(Vo, out["V_out"])
+
+
+def test_compress_per_layer_equals_step_api(kernel_path):
+    """Per-layer ranking in the fused pass (which scores and ranks only the
+    layers the budgets keep) gives the step API's result bit for bit."""
+    L, Hq, Hkv, d, n, W, rr = 6, 8, 2, 128, 1500, 16, (28, 100)
+    Q, K, V = (_rand(s, 950 + i, torch.bfloat16).to(DEV) for i, s in
+               enumerate([(L, Hq, W, d), (L, Hkv, n, d), (L, Hkv, n, d)], 1))
+    B, Nq, h = vc.viscache_plan_budgets(L, n, *rr)
+    assert B[-1] == 0                                    # an evicted layer
+    ref = run_steps(Q, K, V, B, Nq, rank_mode=vc.VC_RANK_PER_LAYER)
+    batch = vc.Batch([n], [W], [rr])
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16, rank_mode=vc.VC_RANK_PER_LAYER)
+    Ko, Vo, idx = vc.prunekv_compress(batch, prm, Q, K, V)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, ref["keep"]) and torch.equal(Ko, ref["K_out"])
+    assert torch.equal(Vo, ref["V_out"])

@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
                     help="layer-budget schedule (the paper's ablation axes); parabola is the method")
+    ap.add_argument("--stage", choices=["prunekv", "scout"], default="prunekv",
+                    help="prunekv: the compression pass (the headline); scout: MMR keyframe selection")
     ap.add_argument("--rank", choices=["shared", "per_layer"], default="shared",
                     help="ranking: one order per KV head from the layer mean (method default) or per layer")
     ap.add_argument("--drop", choices=["survivors", "all"], default="survivors",
@@ -275,8 +277,108 @@ def workload_config(wl, args=None):
             "l2": "inputs larger than L2 (%.2f GB of Qw+K+V > 129 MB)" % (in_bytes / 1e9)}
 
 
+def run_scout(args):
+    """--stage scout: Eq. (mmr) keyframe selection on a batch of synthetic videos."""
+    import torch
+    from fractions import Fraction
+
+    from oracle import scout as osc
+    from paper_2608_24063_gb300 import synth
+    from paper_2608_24063_gb300 import viscache as vc
+
+    n_vid, F, D, lam, p = 64, 64, 512, 0.7, (3, 4)
+    vids = [synth.scout_embeddings(1000 + i, F, D) for i in range(n_vid)]
+    cfg = {"workload": "scout: %d videos x %d frames, D=%d (CLIP ViT-B/32 width), lambda=%.1f, p=%d/%d"
+           % (n_vid, F, D, lam, p[0], p[1]), "videos": n_vid, "frames": F, "D": D}
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        for _ in range(args.warmup):
+            osc.scout(vids[0][0].double().numpy(), vids[0][1].double().numpy(), lam, Fraction(*p))
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            h, t = vids[i % n_vid]
+            osc.scout(h.double().numpy(), t.double().numpy(), lam, Fraction(*p))
+        dt = (time.perf_counter() - t0) / args.steps
+        val = 1.0 / dt
+        print(json.dumps({"metric": "scout keyframe selection videos/s", "value": val, "unit": "videos/s",
+                          "impl": "reference", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+                          "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+                          "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": cfg,
+                          "cpu_baseline": {"value": val, "unit": "videos/s", "cores": cpu_cores(),
+                                           "kind": "oracle", "sample": "one video per step"},
+                          "e2e": {"value": val, "unit": "videos/s", "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}))
+        return
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    H = torch.cat([h for h, _ in vids]).to(dev)
+    T = torch.stack([t for _, t in vids]).to(dev)
+    sizes = [F] * n_vid
+    o0, k0, g0, _ = vc.viscache_scout_mmr(H, T, sizes, lam, p)
+    nf = (__import__("ctypes").c_int32 * n_vid)(*sizes)
+    wsb = torch.empty(max(vc.lib().viscache_scout_workspace_size(n_vid, nf, D), 256), dtype=torch.uint8,
+                      device=dev)
+
+    def step():
+        return vc.viscache_scout_mmr(H, T, sizes, lam, p, out=(o0, k0, g0), ws=wsb)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    vc.viscache_profile_enable(True)
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize()
+    kern = {k: v[0] / v[1] for k, v in vc.viscache_profile_read().items()}
+    vc.viscache_profile_enable(False)
+    # end to end: embeddings from pinned host memory, keyframes back to the host
+    hH, hT = H.cpu().pin_memory(), T.cpu().pin_memory()
+    a.record()
+    for _ in range(args.steps):
+        order, keys, gains, ks = vc.viscache_scout_mmr(hH.to(dev, non_blocking=True),
+                                                       hT.to(dev, non_blocking=True), sizes, lam, p,
+                                                       out=(o0, k0, g0), ws=wsb)
+        keys.cpu()
+    b.record()
+    torch.cuda.synchronize()
+    ems = a.elapsed_time(b) / args.steps
+    # the oracle on the host cores, a bounded sample
+    t0 = time.perf_counter()
+    nv = 0
+    while time.perf_counter() - t0 < min(args.cpu_seconds, 5.0) or nv == 0:
+        h, t = vids[nv % n_vid]
+        osc.scout(h.double().numpy(), t.double().numpy(), lam, Fraction(*p))
+        nv += 1
+    cpu = nv / (time.perf_counter() - t0)
+    k = ks[0]
+    print(json.dumps({
+        "metric": "scout keyframe selection videos/s", "value": n_vid / (ms * 1e-3), "unit": "videos/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded scene-structured embeddings)", "config": cfg,
+        "kernels_ms_per_step": kern, "gpu_launches": len(kern) * args.steps,
+        "picks_per_video": k, "kernel_us_per_batch": sum(kern.values()) * 1e3,
+        "cpu_baseline": {"value": cpu, "unit": "videos/s", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": "%d videos, one at a time (fp64 numpy)" % nv},
+        "e2e": {"value": n_vid / (ems * 1e-3), "unit": "videos/s",
+                "h2d_bytes_per_step": int(hH.numel() * 4 + hT.numel() * 4),
+                "d2h_bytes_per_step": int(keys.numel() * 4)}}))
+
+
 def main():
     args = parse()
+    if args.stage == "scout":
+        run_scout(args)
+        return
     from paper_2608_24063_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
     if args.impl == "reference":

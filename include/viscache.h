@@ -262,6 +262,38 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw,
                      int32_t* idx_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * viscache_scout_mmr -- keyframe selection of the scout stage, Eq. (mmr)
+ * (Sec. 3.1): per video, frames join the selected set Omega greedily by
+ *     lambda * sim(h_f, h_t) - (1 - lambda) * max_{f' in Omega} sim(h_f, h_f')
+ * with sim the cosine similarity, until k = ceil(p * F) frames are chosen
+ * (Sec. 4: lambda = 0.7, p = 0.75).  Readings: the redundancy term is 0 while
+ * Omega is empty (the first pick is the most prompt-relevant frame), ties go
+ * to the lower frame index, a zero vector has similarity 0.  fp32 arithmetic.
+ *
+ *   H             device fp32 [sum_r F_r][D] frame embeddings, video after video
+ *   prompt        device fp32 [n_req][D] prompt embeddings
+ *   n_req         videos, 1..64
+ *   n_frames      host int32 [n_req]: F_r, 1..4096
+ *   D             embedding width, 1..8192
+ *   lambda        relevance weight in [0, 1]
+ *   p_num/p_den   frame retention ratio p in (0, 1]
+ *   order_out     device int32 [sum_r k_r]: picks in selection order, video r
+ *                 at row sum_{r'<r} k_r'
+ *   keyframes_out device int32, same rows: the picks in ascending frame order
+ *   gains_out     device fp32, same rows (nullable): each pick's MMR score
+ *   k_out         host int32 [n_req] (nullable): k_r
+ *   ws            device workspace, 256-byte aligned, viscache_scout_workspace_size bytes
+ * All outputs and ws are caller-owned; the call is asynchronous on `stream`.
+ * Errors: VC_ERR_INVALID_ARG (sizes, ranges, NULL or misaligned inputs),
+ * VC_ERR_WORKSPACE, VC_ERR_CUDA.
+ */
+size_t viscache_scout_workspace_size(int32_t n_req, const int32_t* n_frames, int32_t D);
+int viscache_scout_mmr(const float* H, const float* prompt, int32_t n_req, const int32_t* n_frames,
+                       int32_t D, float lambda, uint32_t p_num, uint32_t p_den, int32_t* order_out,
+                       int32_t* keyframes_out, float* gains_out, int32_t* k_out, void* ws,
+                       size_t ws_bytes, void* stream);
+
+/*
  * prunekv_get_status -- device-side status of the last call that used ws.
  * Synchronises the stream, returns VC_OK or the first device error code
  * recorded (VC_ERR_DEVICE_TIMEOUT, VC_ERR_DEVICE_INDEX), or VC_ERR_CUDA.

@@ -36,6 +36,7 @@ _IH_SCALE = math.sqrt(3.0) / 65536.0
 
 # Stream tags: one independent stream per tensor kind.
 TAG_Q, TAG_K, TAG_V, TAG_CHOICE = 1, 2, 3, 4
+TAG_SCOUT = 5
 
 
 def _signed(u: int) -> int:
@@ -322,3 +323,23 @@ def generate(wl: Workload, device="cpu"):
         ks.append(k)
         vs.append(v)
     return qs, ks, vs
+
+
+# ---------------------------------------------------------------------------
+# Scout inputs: frame and prompt embeddings (stand-ins for CLIP ViT-B/32
+# outputs, width 512).  A video is a run of scenes; a frame is its scene's
+# centre plus per-frame noise (consecutive frames of a scene are near
+# duplicates), and the prompt sits near the centre of one scene.  No MMR
+# arithmetic here.
+
+def scout_embeddings(seed: int, F: int, D: int = 512, noise: float = 0.5,
+                     scene_len: int = 8) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(H [F][D] fp32, prompt [D] fp32) on the CPU, the same bits every time."""
+    n_scenes = (F + scene_len - 1) // scene_len
+    centres = normal(stream_key(TAG_SCOUT, seed, 0), 0, n_scenes * D, "cpu").view(n_scenes, D)
+    eps = normal(stream_key(TAG_SCOUT, seed, 1), 0, F * D, "cpu").view(F, D)
+    scene = torch.arange(F) // scene_len
+    H = centres[scene] + noise * eps
+    target = _Choices(stream_key(TAG_SCOUT, seed, 2)).randint(0, n_scenes - 1)
+    prompt = centres[target] + noise * normal(stream_key(TAG_SCOUT, seed, 3), 0, D, "cpu")
+    return H.to(torch.float32), prompt.to(torch.float32)

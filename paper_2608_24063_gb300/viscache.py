@@ -39,7 +39,7 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
             "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
-            "viscache_device_accessible")
+            "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr")
 
 
 class VisCacheError(RuntimeError):
@@ -77,6 +77,9 @@ def lib() -> ctypes.CDLL:
         L.viscache_plan_budgets.argtypes = [i32, i32, u32, u32, i32, u32, u32, pi32, pi32, pi32]
         L.viscache_plan_budgets_ex.argtypes = [i32, i32, u32, u32, i32, u32, u32, i32, i32, pi32, pi32,
                                                pi32]
+        L.viscache_scout_workspace_size.argtypes = [i32, pi32, i32]
+        L.viscache_scout_workspace_size.restype = sz
+        L.viscache_scout_mmr.argtypes = [vp, vp, i32, pi32, i32, f32, u32, u32, vp, vp, vp, pi32, vp, sz, vp]
         L.prunekv_score_workspace_size.argtypes = [i32, i32, i32]
         L.prunekv_score_workspace_size.restype = sz
         L.prunekv_score.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp, vp,
@@ -174,6 +177,42 @@ def viscache_plan_budgets_ex(L: int, n_vis: int, rr_num: int, rr_den: int, h: in
            lib().viscache_plan_budgets_ex(L, n_vis, rr_num, rr_den, h, m_num, m_den, schedule,
                                           drop_mode, B, ctypes.byref(nq), ctypes.byref(hh)))
     return list(B), nq.value, hh.value
+
+
+def viscache_scout_mmr(H: torch.Tensor, prompt: torch.Tensor, n_frames: Sequence[int], lam: float = 0.7,
+                       p: Tuple[int, int] = (3, 4), with_gains: bool = True, stream=None,
+                       out: Optional[Tuple[torch.Tensor, torch.Tensor, Optional[torch.Tensor]]] = None,
+                       ws: Optional[torch.Tensor] = None):
+    """Keyframe selection, Eq. (mmr): returns (order, keyframes, gains, k per video).
+
+    H: device fp32 [sum F][D], prompt: device fp32 [n_req][D].  ``out`` may
+    hold preallocated (order, keyframes, gains) int32/int32/fp32 [sum k]
+    tensors and ``ws`` a workspace, so repeated calls allocate nothing.
+    """
+    n_req = len(n_frames)
+    D = H.shape[1]
+    nf = (ctypes.c_int32 * n_req)(*n_frames)
+    need = lib().viscache_scout_workspace_size(n_req, nf, D)
+    if need == 0:
+        raise VisCacheError("viscache_scout_workspace_size", VC_ERR_INVALID_ARG)
+    ks = [max(1, min(f, (p[0] * f + p[1] - 1) // p[1])) for f in n_frames]
+    dev = H.device
+    if out is not None:
+        order, keys, gains = out
+    else:
+        order = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+        keys = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+        gains = torch.empty(sum(ks), dtype=torch.float32, device=dev) if with_gains else None
+    ws = _workspace(need, dev, ws)
+    k_out = (ctypes.c_int32 * n_req)()
+    if H.dtype != torch.float32 or prompt.dtype != torch.float32 or not H.is_contiguous() \
+            or not prompt.is_contiguous() or prompt.shape != (n_req, D) or H.shape[0] != sum(n_frames):
+        raise VisCacheError("viscache_scout_mmr", VC_ERR_INVALID_ARG)
+    _check("viscache_scout_mmr", lib().viscache_scout_mmr(
+        _ptr(H), _ptr(prompt), n_req, nf, D, float(lam), p[0], p[1], _ptr(order), _ptr(keys),
+        _ptr(gains), k_out, _ptr(ws), ws.numel(), _stream(stream)))
+    assert list(k_out) == ks
+    return order, keys, gains, ks
 
 
 def prunekv_score_workspace_size(L: int, Hq: int, W: int) -> int:

@@ -22,7 +22,9 @@ import pytest
 
 from oracle import plan
 from oracle import prunekv as ok
+from oracle import scout as osc
 from tests import test_oracle_plan as pins_plan
+from tests import test_oracle_scout as pins_scout
 from tests import test_oracle_scores as pins_scores
 from tests import test_oracle_select_fuse as pins_select_fuse
 
@@ -223,7 +225,32 @@ def _plan_total_floor(L, n, rr, h=None, m=Fraction(3, 4), schedule="parabola", d
     return B, (n if drop == "all" else Nq), h
 
 
+def _mmr(H, h_t, lam, k, swap=False, ties_high=False, red_mode="max", unit=True):
+    Hn = osc.cosine_unit(H) if unit else np.asarray(H, dtype=np.float64)
+    tn = osc.cosine_unit(h_t[None, :])[0] if unit else np.asarray(h_t, dtype=np.float64)
+    F = Hn.shape[0]
+    rel = Hn @ tn
+    a, b = (1.0 - lam, lam) if swap else (lam, 1.0 - lam)
+    chosen = np.zeros(F, dtype=bool)
+    order, gains, picked = [], [], []
+    for step in range(k):
+        if picked:
+            sims = Hn @ Hn[picked].T
+            red = {"max": sims.max(axis=1), "mean": sims.mean(axis=1), "last": sims[:, -1]}[red_mode]
+        else:
+            red = np.zeros(F)
+        score = a * rel - b * red
+        score[chosen] = -np.inf
+        f = int(F - 1 - np.argmax(score[::-1])) if ties_high else int(np.argmax(score))
+        order.append(f)
+        gains.append(score[f])
+        chosen[f] = True
+        picked.append(f)
+    return np.array(order, dtype=np.int64), np.array(gains)
+
+
 SCORES = [pins_scores, pins_select_fuse]
+SCOUT = [pins_scout]
 SELECT_FUSE = [pins_select_fuse]
 PLAN = [pins_plan]
 
@@ -278,11 +305,21 @@ MUTATIONS = [
     ("geometric blocks smaller first", plan, "schedule_proportions",
      _schedule_mutant(small_blocks_first=True), PLAN),
     ("drop-all reading ignored", plan, "plan_budgets", _plan_drop_all_ignored, PLAN),
+    # scout keyframe selection (Eq. mmr)
+    ("relevance and redundancy weights swapped", osc, "mmr_select",
+     lambda *a: _mmr(*a, swap=True), SCOUT),
+    ("MMR ties to the higher frame", osc, "mmr_select", lambda *a: _mmr(*a, ties_high=True), SCOUT),
+    ("redundancy as the mean over the selected frames", osc, "mmr_select",
+     lambda *a: _mmr(*a, red_mode="mean"), SCOUT),
+    ("redundancy to the last pick only", osc, "mmr_select", lambda *a: _mmr(*a, red_mode="last"), SCOUT),
+    ("dot products instead of cosines", osc, "mmr_select", lambda *a: _mmr(*a, unit=False), SCOUT),
+    ("keyframe count rounded down", osc, "keyframe_count",
+     lambda F, p: max(1, min(F, floor(Fraction(p) * F))), SCOUT),
 ]
 
 
 def test_pins_pass_on_the_oracle():
-    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse]) == []
+    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse, pins_scout]) == []
 
 
 @pytest.mark.parametrize("what,module,attr,mutant,pins", MUTATIONS, ids=[m[0] for m in MUTATIONS])

@@ -46,7 +46,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
                     help="layer-budget schedule (the paper's ablation axes); parabola is the method")
-    ap.add_argument("--stage", choices=["prunekv", "scout"], default="prunekv",
+    ap.add_argument("--stage", choices=["prunekv", "scout", "decode"], default="prunekv",
                     help="prunekv: the compression pass (the headline); scout: MMR keyframe selection")
     ap.add_argument("--rank", choices=["shared", "per_layer"], default="shared",
                     help="ranking: one order per KV head from the layer mean (method default) or per layer")
@@ -374,10 +374,195 @@ def run_scout(args):
                 "d2h_bytes_per_step": int(keys.numel() * 4)}}))
 
 
+def run_decode(args):
+    """--stage decode: one decode step's attention in every layer over the
+    compressed cache (the pass's output layout) and, for comparison, over the
+    full cache (every B_l = n, the same kernels)."""
+    import torch
+
+    from oracle import decode as odec
+    from paper_2608_24063_gb300 import viscache as vc
+
+    n_req, L, Hq, Hkv, d, n, T, rr = 16, 28, 28, 4, 128, 12544, 512, (19, 100)
+    cfg = {"workload": "decode step, %d requests on the 7B shape (L=%d, Hq=%d, Hkv=%d, d=%d, bf16), "
+                       "n=%d visual + T=%d text tokens, RR=%d%%" % (n_req, L, Hq, Hkv, d, n, T, rr[0]),
+           "requests": n_req, "L": L, "Hq": Hq, "Hkv": Hkv, "d": d, "n_vis": n, "text": T,
+           "retention": "%d/%d" % rr, "schedule": "parabola"}
+    metric = "decode-step attention tokens/s over the compressed visual cache (all layers)"
+    batch_c = vc.Batch([n] * n_req, [64] * n_req, [rr] * n_req)
+    prm_c = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    B, _, _ = vc.viscache_plan_budgets(L, n, *rr)
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        import numpy as np
+        rng = np.random.default_rng(5)
+        Kc = [rng.standard_normal((Hkv, b, d)) for b in B]
+        Vc = [rng.standard_normal((Hkv, b, d)) for b in B]
+        Kt, Vt = rng.standard_normal((Hkv, T, d)), rng.standard_normal((Hkv, T, d))
+        q = rng.standard_normal((Hq, d))
+
+        def one_request():
+            for l in range(L):
+                odec.decode_attention(q, Kc[l], Vc[l], Kt, Vt)
+
+        for _ in range(args.warmup):
+            one_request()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            one_request()
+        dt = (time.perf_counter() - t0) / args.steps
+        val = 1.0 / dt
+        print(json.dumps({"metric": metric, "value": val, "unit": "tokens/s", "impl": "reference",
+                          "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+                          "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+                          "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": cfg,
+                          "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cpu_cores(),
+                                           "kind": "oracle", "sample": "one request's step (all layers) per step"},
+                          "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}))
+        return
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(12544)
+
+    def normal(*shape):
+        return torch.empty(shape, dtype=torch.bfloat16, device=dev).normal_(generator=gen)
+
+    batch_f = vc.Batch([n] * n_req, [64] * n_req, [(1, 1)] * n_req)
+    prm_f = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16, h=L, m=(1, 1), schedule=vc.VC_SCHED_FIXED)
+    rows_c = vc.compressed_rows(batch_c, prm_c)
+    texts = [T] * n_req
+    caches = {"compressed": (batch_c, prm_c, normal(rows_c, d), normal(rows_c, d)),
+              "full": (batch_f, prm_f, normal(n_req * L * Hkv * n, d), normal(n_req * L * Hkv * n, d))}
+    Kt, Vt = normal(L, n_req * Hkv * T, d), normal(L, n_req * Hkv * T, d)
+    q = normal(L, n_req, Hq, d)
+    out = torch.empty_like(q)
+    ws = torch.empty(max(vc.viscache_decode_workspace_size(b, p, texts) for b, p, _, _ in caches.values()),
+                     dtype=torch.uint8, device=dev)
+
+    def step(name, qq=q):
+        b, p, K, V = caches[name]
+        for l in range(L):
+            vc.viscache_decode_attention(b, p, l, qq[l], K, V, Kt[l], Vt[l], texts, out=out[l], ws=ws)
+
+    res = {}
+    clk = None
+    for name in ("full", "compressed"):
+        for _ in range(max(3, args.warmup)):
+            step(name)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            step(name)
+            with torch.cuda.graph(g):
+                step(name)
+        torch.cuda.current_stream().wait_stream(s)
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if name == "compressed":
+            clocks = ClockSampler(local)
+            clocks.start()
+        a.record()
+        for _ in range(args.steps):
+            g.replay()
+        b.record()
+        torch.cuda.synchronize()
+        if name == "compressed":
+            clk = clocks.stop()
+        ms = a.elapsed_time(b) / args.steps
+        vc.viscache_profile_enable(True)
+        for _ in range(args.steps):
+            step(name)
+        torch.cuda.synchronize()
+        prof = vc.viscache_profile_read()
+        kern = {k: v[0] / args.steps for k, v in prof.items()}
+        launches = {k: v[1] // args.steps for k, v in prof.items()}
+        vc.viscache_profile_enable(False)
+        del g
+        res[name] = (ms, kern, launches)
+    ms, kern, launches = res["compressed"]
+    ms_full, kern_full, _ = res["full"]
+    # algorithmic bytes of a step: every cached K and V row of every layer once,
+    # plus the query rows (decode_partial, L launches a step); achieved =
+    # those bytes over the launches' summed event time
+    kv_rows = sum(n_req * Hkv * (b + T) for b in B)
+    kv_rows_full = L * n_req * Hkv * (n + T)
+    q_bytes = L * n_req * Hq * d * 2
+    pk = peaks()
+    t_part = kern.get("decode_partial", float("nan")) * 1e-3
+    achieved = (kv_rows * d * 2 * 2 + q_bytes) / t_part / 1e9
+    t_part_f = kern_full.get("decode_partial", float("nan")) * 1e-3
+    achieved_f = (kv_rows_full * d * 2 * 2 + q_bytes) / t_part_f / 1e9
+    # end to end through the public call: this step's query rows from pinned
+    # host memory, the attention outputs back to the host
+    hq = q.cpu().pin_memory()
+    hout = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    qd = torch.empty_like(q)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for _ in range(2):
+        qd.copy_(hq, non_blocking=True)
+        step("compressed", qd)
+        hout.copy_(out, non_blocking=True)
+    torch.cuda.synchronize()
+    a.record()
+    for _ in range(args.steps):
+        qd.copy_(hq, non_blocking=True)
+        step("compressed", qd)
+        hout.copy_(out, non_blocking=True)
+    b.record()
+    torch.cuda.synchronize()
+    ems = a.elapsed_time(b) / args.steps
+    # the oracle on the host cores: one request's step over every layer
+    import numpy as np
+    Kc, Vc = caches["compressed"][2], caches["compressed"][3]
+    Kn = [Kc[Hkv * sum(B[:l]):Hkv * sum(B[:l + 1])].double().cpu().numpy().reshape(Hkv, B[l], d) for l in range(L)]
+    Vn = [Vc[Hkv * sum(B[:l]):Hkv * sum(B[:l + 1])].double().cpu().numpy().reshape(Hkv, B[l], d) for l in range(L)]
+    Ktn = [Kt[l, :Hkv * T].double().cpu().numpy().reshape(Hkv, T, d) for l in range(L)]
+    Vtn = [Vt[l, :Hkv * T].double().cpu().numpy().reshape(Hkv, T, d) for l in range(L)]
+    qn = q[:, 0].double().cpu().numpy()
+    t0 = time.perf_counter()
+    nr = 0
+    while time.perf_counter() - t0 < min(args.cpu_seconds, 10.0) or nr == 0:
+        for l in range(L):
+            odec.decode_attention(qn[l], Kn[l], Vn[l], Ktn[l], Vtn[l])
+        nr += 1
+    cpu = nr / (time.perf_counter() - t0)
+    print(json.dumps({
+        "metric": metric, "value": n_req / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded normal cache)",
+        "config": dict(cfg, launch="cuda graph of the %d per-layer calls" % L,
+                       l2="a step reads %.2f GB of cache > 129 MB L2" % (kv_rows * d * 4 / 1e9)),
+        "full_cache": {"ms_per_step": ms_full, "value": n_req / (ms_full * 1e-3),
+                       "speedup_of_compressed": ms_full / ms,
+                       "kernels_ms_per_step": kern_full,
+                       "partial_gbs": achieved_f},
+        "kernels_ms_per_step": kern,
+        "roofline": {"kernel": "decode_partial", "bound": "hbm", "achieved": achieved,
+                     "peak": pk["hbm"], "unit": "GB/s", "frac": achieved / pk["hbm"], "traffic": None,
+                     "peak_source": pk["source"]},
+        "cpu_baseline": {"value": cpu, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": "%d single-request steps over all %d layers (fp64 numpy)" % (nr, L)},
+        "e2e": {"value": n_req / (ems * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(q.numel() * 2), "d2h_bytes_per_step": int(out.numel() * 2)},
+        "gpu_launches": sum(launches.values()) * args.steps, "clocks": clk}))
+
+
 def main():
     args = parse()
     if args.stage == "scout":
         run_scout(args)
+        return
+    if args.stage == "decode":
+        run_decode(args)
         return
     from paper_2608_24063_gb300 import synth
     wl = synth.WORKLOADS[args.workload]

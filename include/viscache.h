@@ -315,6 +315,41 @@ int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* lau
                           int max_kernels);
 
 /*
+ * viscache_decode_attention -- one decode step's attention in layer `layer`
+ * over the cache that prunekv_compress left (Sec. 2 "VLLM Decoding"; after
+ * PruneKV, Sec. 3.2, the visual part of layer l holds B_l rows per KV head):
+ *     out[r][j] = softmax(q[r][j] . K_g^T * scale) V_g,   g = j / (Hq / Hkv),
+ * over request r's B_l kept visual rows of KV head g followed by its T_r text
+ * rows.  fp32 accumulation, out rounded once to the input type.
+ *
+ *   batch, p      the batch and parameters prunekv_compress ran with (they fix
+ *                 every B_l); 1..256 requests, Hq / Hkv <= 8
+ *   layer         0..L-1
+ *   q             device [n_req][Hq][d], the step's query rows
+ *   K_out, V_out  device [rows][d]: prunekv_compress's outputs; layer l, KV
+ *                 head g of request r at row R_r + Hkv * P_l + g * B_l with
+ *                 P_l = sum_{l'<l} B_l' and R_r = sum_{r'<r} Hkv * sum_l B_l
+ *                 (a full cache in [L][Hkv][n][d] order per request is this
+ *                 layout with every B_l = n)
+ *   K_text, V_text device [sum_r Hkv * T_r][d], this layer's text rows, per
+ *                 request [Hkv][T_r][d] packed; NULL when n_text is NULL
+ *   n_text        host int32 [n_req] (nullable = no text): T_r, 0..2^24
+ *   out           device [n_req][Hq][d]; a query with no keys gets zeros
+ *   ws            device workspace, 256-byte aligned,
+ *                 viscache_decode_workspace_size bytes (enough for any layer)
+ * Types follow p->dtype (bf16 or fp32); every pointer 16-byte aligned.  All
+ * buffers are caller-owned; the call is asynchronous on `stream`.
+ * Errors: VC_ERR_INVALID_ARG (shapes, ranges, NULL or misaligned pointers),
+ * VC_ERR_WORKSPACE, VC_ERR_CUDA.
+ */
+size_t viscache_decode_workspace_size(const vc_batch* batch, const vc_params* p,
+                                      const int32_t* n_text);
+int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t layer,
+                              const void* q, const void* K_out, const void* V_out,
+                              const void* K_text, const void* V_text, const int32_t* n_text,
+                              void* out, void* ws, size_t ws_bytes, void* stream);
+
+/*
  * Kernel path selection (process-wide, default VC_PATH_AUTO): AUTO runs the
  * score (Eq. token_score) and the fusion (Eq. redistribution, weight_fusion)
  * of bf16, d = 128 problems on the tcgen05 tensor cores and everything else

@@ -404,6 +404,55 @@ Layout compress_layout(const vc_params* p, const std::vector<RequestPlan>& plans
   return lay;
 }
 
+// Decode table of one layer: request r's visual rows start at
+// R_r + Hkv * P_l (R_r = rows of the earlier requests, P_l = sum of the
+// earlier layers' budgets); its text rows at Hkv * (sum of earlier T).
+// Returns VC_ERR_INVALID_ARG when the batch does not fit the table.
+int decode_table(const vc_params* p, const std::vector<RequestPlan>& plans, int layer,
+                 const int32_t* n_text, DecodeTable* tb) {
+  const int n_req = (int)plans.size();
+  if (n_req > kDecodeMaxReq || p->Hq / p->Hkv > kDecodeMaxGroup) return VC_ERR_INVALID_ARG;
+  tb->n_req = n_req; tb->Hq = p->Hq; tb->Hkv = p->Hkv; tb->G = p->Hq / p->Hkv;
+  tb->scale = p->scale == 0.f ? 1.0f / sqrtf((float)p->d) : p->scale;
+  const int64_t split = decode_split_keys();
+  int64_t rows = 0, text = 0, units = 0;
+  for (int r = 0; r < n_req; ++r) {
+    const RequestPlan& pl = plans[r];
+    const int32_t T = n_text ? n_text[r] : 0;
+    if (T < 0 || T > (1 << 24)) return VC_ERR_INVALID_ARG;
+    int64_t P = 0, all = 0;
+    for (int l = 0; l < p->L; ++l) {
+      if (l < layer) P += pl.B[l];
+      all += pl.B[l];
+    }
+    DecodeReq& q = tb->req[r];
+    q.vis_row0 = rows + (int64_t)p->Hkv * P;
+    q.txt_row0 = text;
+    q.B = pl.B[layer];
+    q.T = T;
+    q.unit0 = (int32_t)units;
+    q.nsplit = (int32_t)((q.B + (int64_t)T + split - 1) / split);
+    units += (int64_t)p->Hkv * q.nsplit;
+    if (units > (int64_t)1 << 30) return VC_ERR_INVALID_ARG;
+    rows += (int64_t)p->Hkv * all;
+    text += (int64_t)p->Hkv * T;
+  }
+  tb->units = (int32_t)units;
+  return VC_OK;
+}
+
+struct DecodeWs {
+  size_t o_ml = 0, o_o = 0, total = 0;
+};
+DecodeWs decode_ws(int64_t units, int d) {
+  Arena a;
+  DecodeWs w;
+  w.o_ml = a.take(sizeof(float2) * kDecodeMaxGroup * std::max<int64_t>(units, 1));
+  w.o_o = a.take(sizeof(float) * kDecodeMaxGroup * d * std::max<int64_t>(units, 1));
+  w.total = a.off;
+  return w;
+}
+
 }  // namespace
 }  // namespace vc
 
@@ -554,6 +603,45 @@ int prunekv_get_status(const void* ws, void* stream) {
     return VC_ERR_CUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return VC_ERR_CUDA;
   return s;
+}
+
+size_t viscache_decode_workspace_size(const vc_batch* batch, const vc_params* p,
+                                      const int32_t* n_text) {
+  std::vector<RequestPlan> plans;
+  if (plan_batch(batch, p, &plans) != VC_OK) return 0;
+  static thread_local DecodeTable tb;
+  int64_t units = 0;
+  for (int l = 0; l < p->L; ++l) {
+    if (decode_table(p, plans, l, n_text, &tb) != VC_OK) return 0;
+    units = std::max<int64_t>(units, tb.units);
+  }
+  return decode_ws(units, p->d).total;
+}
+
+int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t layer,
+                              const void* q, const void* K_out, const void* V_out,
+                              const void* K_text, const void* V_text, const int32_t* n_text,
+                              void* out, void* ws, size_t ws_bytes, void* stream) {
+  std::vector<RequestPlan> plans;
+  const int rc = plan_batch(batch, p, &plans);
+  if (rc != VC_OK) return rc;
+  if (layer < 0 || layer >= p->L) return VC_ERR_INVALID_ARG;
+  if (!q || !K_out || !V_out || !out || !aligned16(q) || !aligned16(K_out) || !aligned16(V_out) ||
+      !aligned16(out))
+    return VC_ERR_INVALID_ARG;
+  if (n_text && (!K_text || !V_text || !aligned16(K_text) || !aligned16(V_text)))
+    return VC_ERR_INVALID_ARG;
+  static thread_local DecodeTable tb;
+  const int tc = decode_table(p, plans, layer, n_text, &tb);
+  if (tc != VC_OK) return tc;
+  const DecodeWs dw = decode_ws(tb.units, p->d);
+  const int wc = check_ws(ws, ws_bytes, dw.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  return cuda_status(launch_decode(tb, p->dtype, p->d, q, K_out, V_out, K_text, V_text, out,
+                                   reinterpret_cast<float*>(w + dw.o_o),
+                                   reinterpret_cast<float2*>(w + dw.o_ml),
+                                   static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

@@ -66,4 +66,28 @@ cudaError_t launch_fuse_simt(int dtype, const void* V, const Shape& sh, const Ta
                              const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
                              void* V_out, int units, cudaStream_t st);
 
+// Decode attention over the compressed cache of one layer (Sec. 2, after
+// Sec. 3.2): per (request, KV head) the layer's B kept visual rows (dense
+// varlen layout of prunekv_compress) then T text rows, split into chunks of
+// decode_split_keys() keys; partial softmax states are merged per query head.
+constexpr int kDecodeMaxReq = 256;
+constexpr int kDecodeMaxGroup = 8;            // query heads per KV head
+struct DecodeReq {
+  int64_t vis_row0;        // first visual row of KV head 0 (rows g*B ... of head g)
+  int64_t txt_row0;        // first text row of KV head 0 (rows g*T ... of head g)
+  int32_t B, T;            // visual and text rows per KV head
+  int32_t unit0;           // first (KV head, split) unit of the request
+  int32_t nsplit;          // splits per KV head, ceil((B+T) / split keys)
+};
+struct DecodeTable {
+  int32_t n_req, Hq, Hkv, G;
+  float scale;
+  int32_t units;           // sum over requests of Hkv * nsplit
+  DecodeReq req[kDecodeMaxReq];
+};
+int decode_split_keys();
+cudaError_t launch_decode(const DecodeTable& tb, int dtype, int d, const void* q, const void* Kc,
+                          const void* Vc, const void* Kt, const void* Vt, void* out, float* part_o,
+                          float2* part_ml, cudaStream_t st);
+
 }  // namespace vc

@@ -39,7 +39,8 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
             "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
-            "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr")
+            "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr",
+            "viscache_decode_workspace_size", "viscache_decode_attention")
 
 
 class VisCacheError(RuntimeError):
@@ -80,6 +81,10 @@ def lib() -> ctypes.CDLL:
         L.viscache_scout_workspace_size.argtypes = [i32, pi32, i32]
         L.viscache_scout_workspace_size.restype = sz
         L.viscache_scout_mmr.argtypes = [vp, vp, i32, pi32, i32, f32, u32, u32, vp, vp, vp, pi32, vp, sz, vp]
+        L.viscache_decode_workspace_size.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), pi32]
+        L.viscache_decode_workspace_size.restype = sz
+        L.viscache_decode_attention.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), i32,
+                                                vp, vp, vp, vp, vp, pi32, vp, vp, sz, vp]
         L.prunekv_score_workspace_size.argtypes = [i32, i32, i32]
         L.prunekv_score_workspace_size.restype = sz
         L.prunekv_score.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp, vp,
@@ -361,6 +366,32 @@ def prunekv_compress(batch: Batch, params: vc_params, Qw: torch.Tensor, K: torch
         ctypes.byref(batch.c), ctypes.byref(params), _ptr(Qw), _ptr(K), _ptr(V), _ptr(K_out),
         _ptr(V_out), _ptr(idx_out), _ptr(ws), ws.numel(), _stream(stream)))
     return K_out[:rows], V_out[:rows], idx_out[:rows]
+
+
+def viscache_decode_workspace_size(batch: Batch, params: vc_params,
+                                   n_text: Optional[Sequence[int]] = None) -> int:
+    return lib().viscache_decode_workspace_size(ctypes.byref(batch.c), ctypes.byref(params),
+                                                _i32(n_text) if n_text is not None else None)
+
+
+def viscache_decode_attention(batch: Batch, params: vc_params, layer: int, q: torch.Tensor,
+                              K_out: torch.Tensor, V_out: torch.Tensor,
+                              K_text: Optional[torch.Tensor] = None, V_text: Optional[torch.Tensor] = None,
+                              n_text: Optional[Sequence[int]] = None, out: Optional[torch.Tensor] = None,
+                              ws: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """One decode step's attention in `layer` over the compressed cache: q [n_req][Hq][d] -> out."""
+    if out is None:
+        out = torch.empty_like(q)
+    nt = _i32(n_text) if n_text is not None else None
+    if ws is None:
+        need = lib().viscache_decode_workspace_size(ctypes.byref(batch.c), ctypes.byref(params), nt)
+        if need == 0:
+            raise VisCacheError("viscache_decode_workspace_size", VC_ERR_INVALID_ARG)
+        ws = _workspace(need, q.device, None)
+    _check("viscache_decode_attention", lib().viscache_decode_attention(
+        ctypes.byref(batch.c), ctypes.byref(params), int(layer), _ptr(q), _ptr(K_out), _ptr(V_out),
+        _ptr(K_text), _ptr(V_text), nt, _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
+    return out
 
 
 def viscache_set_kernel_path(path: int) -> None:

@@ -136,3 +136,35 @@ def test_workspace_sizes_are_positive_and_aligned():
     prm = vc.make_params(28, 28, 4, 128, vc.VC_BF16)
     assert vc.prunekv_workspace_size(b, prm) > vc.prunekv_score_workspace_size(28, 28, 64)
     assert vc.compressed_rows(b, prm) == 4 * 66734
+
+
+def test_decode_entry_rejects_bad_arguments_without_touching_the_device():
+    lib = vc.lib()
+    p = ctypes.c_void_p(256)
+    b = vc.Batch([100, 50], [8, 8], [(25, 100), (25, 100)])
+    prm = vc.make_params(4, 8, 2, 128, vc.VC_BF16)
+    call = lambda prm, layer, q=p, nt=None, ws=p, wsb=1 << 30: lib.viscache_decode_attention(
+        ctypes.byref(b.c), ctypes.byref(prm), layer, q, p, p, None, None, nt, p, ws, wsb, None)
+    assert call(prm, 4) == vc.VC_ERR_INVALID_ARG                           # layer out of range
+    assert call(prm, -1) == vc.VC_ERR_INVALID_ARG
+    assert call(prm, 0, q=ctypes.c_void_p(264)) == vc.VC_ERR_INVALID_ARG   # misaligned q
+    nt = (ctypes.c_int32 * 2)(3, 0)
+    assert call(prm, 0, nt=nt) == vc.VC_ERR_INVALID_ARG                    # text lengths, no text rows
+    assert call(prm, 0, wsb=16) == vc.VC_ERR_WORKSPACE
+    assert call(prm, 0, ws=ctypes.c_void_p(272)) == vc.VC_ERR_WORKSPACE
+    wide = vc.make_params(4, 32, 2, 128, vc.VC_BF16)                     # 16 query heads per KV head
+    assert call(wide, 0) == vc.VC_ERR_INVALID_ARG
+    assert vc.viscache_decode_workspace_size(b, wide) == 0
+
+
+def test_decode_workspace_covers_every_layer():
+    # the largest layer budget, split into 512-key pieces per KV head, bounds
+    # the partial states (8 query slots x d floats + 8 (max, sum) pairs each)
+    b = vc.Batch([12544], [64], [(19, 100)])
+    prm = vc.make_params(28, 28, 4, 128, vc.VC_BF16)
+    B, _, _ = vc.viscache_plan_budgets(28, 12544, 19, 100)
+    units = 4 * -(-(max(B) + 300) // 512)
+    got = vc.viscache_decode_workspace_size(b, prm, [300])
+    assert got % 256 == 0 and got >= units * 8 * (128 * 4 + 8)
+    assert vc.viscache_decode_workspace_size(b, prm) <= got
+    assert vc.viscache_decode_workspace_size(vc.Batch([100] * 257, [8] * 257, [(1, 4)] * 257), prm) == 0

@@ -414,12 +414,16 @@ int decode_table(const vc_params* p, const std::vector<RequestPlan>& plans, int 
   if (n_req > kDecodeMaxReq || p->Hq / p->Hkv > kDecodeMaxGroup) return VC_ERR_INVALID_ARG;
   tb->n_req = n_req; tb->Hq = p->Hq; tb->Hkv = p->Hkv; tb->G = p->Hq / p->Hkv;
   tb->scale = p->scale == 0.f ? 1.0f / sqrtf((float)p->d) : p->scale;
-  const int64_t split = decode_split_keys();
+  for (int r = 0; r < n_req; ++r) {
+    const int32_t T = n_text ? n_text[r] : 0;
+    if (T < 0 || T > (1 << 24)) return VC_ERR_INVALID_ARG;
+  }
+  const int split = decode_split_keys(p->dtype);
+  tb->split = split;
   int64_t rows = 0, text = 0, units = 0;
   for (int r = 0; r < n_req; ++r) {
     const RequestPlan& pl = plans[r];
     const int32_t T = n_text ? n_text[r] : 0;
-    if (T < 0 || T > (1 << 24)) return VC_ERR_INVALID_ARG;
     int64_t P = 0, all = 0;
     for (int l = 0; l < p->L; ++l) {
       if (l < layer) P += pl.B[l];
@@ -431,7 +435,8 @@ int decode_table(const vc_params* p, const std::vector<RequestPlan>& plans, int 
     q.B = pl.B[layer];
     q.T = T;
     q.unit0 = (int32_t)units;
-    q.nsplit = (int32_t)((q.B + (int64_t)T + split - 1) / split);
+    // a pair without keys still gets one (empty) split, whose merge writes zeros
+    q.nsplit = (int32_t)std::max<int64_t>(1, (q.B + (int64_t)T + split - 1) / split);
     units += (int64_t)p->Hkv * q.nsplit;
     if (units > (int64_t)1 << 30) return VC_ERR_INVALID_ARG;
     rows += (int64_t)p->Hkv * all;
@@ -442,11 +447,12 @@ int decode_table(const vc_params* p, const std::vector<RequestPlan>& plans, int 
 }
 
 struct DecodeWs {
-  size_t o_ml = 0, o_o = 0, total = 0;
+  size_t o_arr = 0, o_ml = 0, o_o = 0, total = 0;
 };
-DecodeWs decode_ws(int64_t units, int d) {
+DecodeWs decode_ws(int64_t units, int d, int pairs) {
   Arena a;
   DecodeWs w;
+  w.o_arr = a.take(sizeof(int32_t) * std::max(pairs, 1));
   w.o_ml = a.take(sizeof(float2) * kDecodeMaxGroup * std::max<int64_t>(units, 1));
   w.o_o = a.take(sizeof(float) * kDecodeMaxGroup * d * std::max<int64_t>(units, 1));
   w.total = a.off;
@@ -615,7 +621,7 @@ size_t viscache_decode_workspace_size(const vc_batch* batch, const vc_params* p,
     if (decode_table(p, plans, l, n_text, &tb) != VC_OK) return 0;
     units = std::max<int64_t>(units, tb.units);
   }
-  return decode_ws(units, p->d).total;
+  return decode_ws(units, p->d, batch->n_req * p->Hkv).total;
 }
 
 int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t layer,
@@ -634,13 +640,14 @@ int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t
   static thread_local DecodeTable tb;
   const int tc = decode_table(p, plans, layer, n_text, &tb);
   if (tc != VC_OK) return tc;
-  const DecodeWs dw = decode_ws(tb.units, p->d);
+  const DecodeWs dw = decode_ws(tb.units, p->d, tb.n_req * tb.Hkv);
   const int wc = check_ws(ws, ws_bytes, dw.total);
   if (wc != VC_OK) return wc;
   uint8_t* w = static_cast<uint8_t*>(ws);
   return cuda_status(launch_decode(tb, p->dtype, p->d, q, K_out, V_out, K_text, V_text, out,
                                    reinterpret_cast<float*>(w + dw.o_o),
                                    reinterpret_cast<float2*>(w + dw.o_ml),
+                                   reinterpret_cast<int32_t*>(w + dw.o_arr),
                                    static_cast<cudaStream_t>(stream)));
 }
 

@@ -77,17 +77,18 @@ struct DecodeReq {
   int64_t txt_row0;        // first text row of KV head 0 (rows g*T ... of head g)
   int32_t B, T;            // visual and text rows per KV head
   int32_t unit0;           // first (KV head, split) unit of the request
-  int32_t nsplit;          // splits per KV head, ceil((B+T) / split keys)
+  int32_t nsplit;          // splits per KV head, max(1, ceil((B+T) / split keys))
 };
 struct DecodeTable {
   int32_t n_req, Hq, Hkv, G;
   float scale;
+  int32_t split;           // keys per split (at most decode_split_keys(dtype))
   int32_t units;           // sum over requests of Hkv * nsplit
   DecodeReq req[kDecodeMaxReq];
 };
-int decode_split_keys();
+int decode_split_keys(int dtype);   // the largest split a kernel takes
 cudaError_t launch_decode(const DecodeTable& tb, int dtype, int d, const void* q, const void* Kc,
                           const void* Vc, const void* Kt, const void* Vt, void* out, float* part_o,
-                          float2* part_ml, cudaStream_t st);
+                          float2* part_ml, int32_t* arrivals, cudaStream_t st);
 
 }  // namespace vc

@@ -182,3 +182,22 @@ def test_rejects_bad_arguments():
     with pytest.raises(vc.VisCacheError):       # text lengths without text rows
         vc.viscache_decode_attention(batch, vc.make_params(2, 8, 2, 128, vc.VC_BF16), 0, q, K, K,
                                      n_text=[3])
+
+
+def test_many_splits_merge():
+    # 9000 + 300 keys per KV head: more than 32 splits of the tensor-core
+    # path, so the merge takes its split states 32 at a time
+    L, Hkv, G, d, n, T = 2, 2, 7, 128, 9000, 300
+    K = _rand((L, Hkv, n, d), 61, torch.bfloat16)
+    V = _rand((L, Hkv, n, d), 62, torch.bfloat16)
+    Kt = _rand((Hkv * T, d), 63, torch.bfloat16)
+    Vt = _rand((Hkv * T, d), 64, torch.bfloat16)
+    batch = vc.Batch([n], [8], [(1, 1)])
+    params = vc.make_params(L, G * Hkv, Hkv, d, vc.VC_BF16, h=L, m=(1, 1), schedule=vc.VC_SCHED_FIXED)
+    q = _rand((1, G * Hkv, d), 65, torch.bfloat16)
+    out = vc.viscache_decode_attention(batch, params, 1, q.to(DEV), K.reshape(-1, d).to(DEV),
+                                       V.reshape(-1, d).to(DEV), Kt.to(DEV), Vt.to(DEV), [T])
+    ref = odec.decode_attention(q[0].double().numpy(), K[1].double().numpy(), V[1].double().numpy(),
+                                Kt.double().numpy().reshape(Hkv, T, d), Vt.double().numpy().reshape(Hkv, T, d))
+    err = np.abs(out[0].float().cpu().numpy() - ref)
+    assert (err <= tolerance(torch.bfloat16, ref, float(V.abs().max()))).all()

@@ -4,7 +4,8 @@ Each case replaces one oracle function (on the CPU, for this test only) with
 a copy that carries a single plausible mistake -- a dropped term, a wrong
 sign, index or axis, a transposed or swapped operand, an off-by-one -- and
 runs the pin tests of that part of the oracle (test_oracle_plan,
-test_oracle_scores, test_oracle_select_fuse).  At least one pin must fail.
+test_oracle_scores, test_oracle_select_fuse, test_oracle_scout,
+test_oracle_decode).  At least one pin must fail.
 
 The pins used here check the oracle against things other than itself: values
 and closed forms from the paper, brute force on tiny inputs, invariants, and
@@ -22,7 +23,9 @@ import pytest
 
 from oracle import plan
 from oracle import prunekv as ok
+from oracle import decode as odec
 from oracle import scout as osc
+from tests import test_oracle_decode as pins_decode
 from tests import test_oracle_plan as pins_plan
 from tests import test_oracle_scout as pins_scout
 from tests import test_oracle_scores as pins_scores
@@ -251,6 +254,32 @@ def _mmr(H, h_t, lam, k, swap=False, ties_high=False, red_mode="max", unit=True)
 
 SCORES = [pins_scores, pins_select_fuse]
 SCOUT = [pins_scout]
+DECODE = [pins_decode]
+
+
+def _decode(q, K_vis, V_vis, K_text=None, V_text=None, scale=None, head_map="group", drop_text=False,
+            scale_mode="sqrt", sum_mode="softmax"):
+    """oracle.decode.decode_attention with one planted mistake."""
+    q = np.asarray(q, dtype=np.float64)
+    Hq, d = q.shape
+    Hkv = K_vis.shape[0]
+    G = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / np.sqrt(d) if scale_mode == "sqrt" else 1.0 / d
+    out = np.zeros((Hq, d))
+    for j in range(Hq):
+        g = j // G if head_map == "group" else j % Hkv
+        Ks, Vs = [np.asarray(K_vis[g], np.float64)], [np.asarray(V_vis[g], np.float64)]
+        if K_text is not None and not drop_text:
+            Ks.append(np.asarray(K_text[g], np.float64))
+            Vs.append(np.asarray(V_text[g], np.float64))
+        Kc, Vc = np.concatenate(Ks), np.concatenate(Vs)
+        if Kc.shape[0] == 0:
+            continue
+        x = (Kc @ q[j]) * scale
+        p = np.exp(x - x.max())
+        out[j] = (p / p.sum()) @ Vc if sum_mode == "softmax" else (p / p.shape[0]) @ Vc
+    return out
 SELECT_FUSE = [pins_select_fuse]
 PLAN = [pins_plan]
 
@@ -315,11 +344,18 @@ MUTATIONS = [
     ("dot products instead of cosines", osc, "mmr_select", lambda *a: _mmr(*a, unit=False), SCOUT),
     ("keyframe count rounded down", osc, "keyframe_count",
      lambda F, p: max(1, min(F, floor(Fraction(p) * F))), SCOUT),
+    # decode attention over the compressed cache (Sec. 2 decoding)
+    ("query head j reads KV head j mod Hkv", odec, "decode_attention",
+     lambda *a, **k: _decode(*a, head_map="mod", **k), DECODE),
+    ("text rows left out", odec, "decode_attention", lambda *a, **k: _decode(*a, drop_text=True, **k), DECODE),
+    ("logits scaled by 1/d", odec, "decode_attention", lambda *a, **k: _decode(*a, scale_mode="d", **k), DECODE),
+    ("weights divided by the key count, not their sum", odec, "decode_attention",
+     lambda *a, **k: _decode(*a, sum_mode="count", **k), DECODE),
 ]
 
 
 def test_pins_pass_on_the_oracle():
-    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse, pins_scout]) == []
+    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse, pins_scout, pins_decode]) == []
 
 
 @pytest.mark.parametrize("what,module,attr,mutant,pins", MUTATIONS, ids=[m[0] for m in MUTATIONS])

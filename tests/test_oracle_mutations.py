@@ -5,7 +5,7 @@ a copy that carries a single plausible mistake -- a dropped term, a wrong
 sign, index or axis, a transposed or swapped operand, an off-by-one -- and
 runs the pin tests of that part of the oracle (test_oracle_plan,
 test_oracle_scores, test_oracle_select_fuse, test_oracle_scout,
-test_oracle_decode).  At least one pin must fail.
+test_oracle_decode, test_oracle_quant).  At least one pin must fail.
 
 The pins used here check the oracle against things other than itself: values
 and closed forms from the paper, brute force on tiny inputs, invariants, and
@@ -24,9 +24,11 @@ import pytest
 from oracle import plan
 from oracle import prunekv as ok
 from oracle import decode as odec
+from oracle import quant as oq
 from oracle import scout as osc
 from tests import test_oracle_decode as pins_decode
 from tests import test_oracle_plan as pins_plan
+from tests import test_oracle_quant as pins_quant
 from tests import test_oracle_scout as pins_scout
 from tests import test_oracle_scores as pins_scores
 from tests import test_oracle_select_fuse as pins_select_fuse
@@ -255,6 +257,46 @@ def _mmr(H, h_t, lam, k, swap=False, ties_high=False, red_mode="max", unit=True)
 SCORES = [pins_scores, pins_select_fuse]
 SCOUT = [pins_scout]
 DECODE = [pins_decode]
+QUANT = [pins_quant]
+
+
+def _params_mutant(levels=15, zero_min=False):
+    def group_params(x, axis):
+        x = np.asarray(x, dtype=np.float32)
+        lo = x.min(axis=axis)
+        hi = x.max(axis=axis)
+        if zero_min:
+            lo = np.zeros_like(lo)
+        return ((hi - lo) / np.float32(levels)).astype(np.float32), lo.astype(np.float32)
+    return group_params
+
+
+def _codes_floor(x, scale, lo):
+    x = np.asarray(x, dtype=np.float32)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        q = np.floor((x - lo) / scale)
+    q = np.where(scale > 0, q, 0.0)
+    return np.clip(q, 0, 15).astype(np.uint8)
+
+
+def _pack_swapped(codes):
+    codes = np.asarray(codes, dtype=np.uint8)
+    return (codes[:, 1::2] | (codes[:, 0::2] << 4)).astype(np.uint8)
+
+
+def _keys_one_group(K):
+    K = np.asarray(K, dtype=np.float32)
+    s, m = oq.group_params(K, axis=0)
+    return oq.codes_of(K, s[None, :], m[None, :]), s[None, :], m[None, :]
+
+
+def _values_group64(V):
+    V = np.asarray(V, dtype=np.float32)
+    R, d = V.shape
+    g = V.reshape(R, d // 64, 64)
+    s, m = oq.group_params(g, axis=2)
+    codes = oq.codes_of(g, s[:, :, None], m[:, :, None]).reshape(R, d)
+    return codes, np.repeat(s, 2, axis=1), np.repeat(m, 2, axis=1)
 
 
 def _decode(q, K_vis, V_vis, K_text=None, V_text=None, scale=None, head_map="group", drop_text=False,
@@ -351,11 +393,19 @@ MUTATIONS = [
     ("logits scaled by 1/d", odec, "decode_attention", lambda *a, **k: _decode(*a, scale_mode="d", **k), DECODE),
     ("weights divided by the key count, not their sum", odec, "decode_attention",
      lambda *a, **k: _decode(*a, sum_mode="count", **k), DECODE),
+    # 4-bit quantisation of the compacted cache
+    ("16 levels per step instead of 15", oq, "group_params", _params_mutant(levels=16), QUANT),
+    ("minimum taken as zero", oq, "group_params", _params_mutant(zero_min=True), QUANT),
+    ("codes rounded down", oq, "codes_of", _codes_floor, QUANT),
+    ("odd channel in the low nibble", oq, "pack", _pack_swapped, QUANT),
+    ("one key group per segment", oq, "quantize_keys", _keys_one_group, QUANT),
+    ("value groups of 64 channels", oq, "quantize_values", _values_group64, QUANT),
 ]
 
 
 def test_pins_pass_on_the_oracle():
-    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse, pins_scout, pins_decode]) == []
+    assert _failing_pins([pins_plan, pins_scores, pins_select_fuse, pins_scout, pins_decode,
+                          pins_quant]) == []
 
 
 @pytest.mark.parametrize("what,module,attr,mutant,pins", MUTATIONS, ids=[m[0] for m in MUTATIONS])

@@ -46,7 +46,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
                     help="layer-budget schedule (the paper's ablation axes); parabola is the method")
-    ap.add_argument("--stage", choices=["prunekv", "scout", "decode"], default="prunekv",
+    ap.add_argument("--stage", choices=["prunekv", "scout", "decode", "quant"], default="prunekv",
                     help="prunekv: the compression pass (the headline); scout: MMR keyframe selection")
     ap.add_argument("--requests", type=int, default=16, help="--stage decode: concurrent requests")
     ap.add_argument("--decode-cache", choices=["both", "compressed", "full"], default="both",
@@ -570,8 +570,147 @@ def run_decode(args):
         "gpu_launches": sum(launches.values()) * args.steps, "clocks": clk}))
 
 
+def run_quant(args):
+    """--stage quant: 4-bit quantisation of the compacted cache of 16 requests
+    on the 7B shape (the decode workload's cache), and its reconstruction."""
+    import numpy as np
+    import torch
+
+    from oracle import quant as oq
+    from paper_2608_24063_gb300 import viscache as vc
+
+    n_req, L, Hq, Hkv, d, n, rr = args.requests, 28, 28, 4, 128, 12544, (19, 100)
+    batch = vc.Batch([n] * n_req, [64] * n_req, [rr] * n_req)
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    rows, groups = vc.viscache_kv4_sizes(batch, prm)
+    cfg = {"workload": "4-bit quantisation of the compacted cache: %d requests on the 7B shape "
+                       "(L=%d, Hkv=%d, d=%d, bf16), n=%d, RR=%d%%: %d rows of K and of V"
+                       % (n_req, L, Hkv, d, n, rr[0], rows),
+           "requests": n_req, "rows": rows, "key_groups": groups, "group": oq.GROUP}
+    metric = "compacted KV quantised to 4 bits, input GB/s"
+    in_bytes = 2 * rows * d * 2
+    out_bytes = 2 * rows * d // 2 + groups * d * 8 + rows * (d // 32) * 8
+    rank = int(os.environ.get("RANK", "0"))
+    sample_rows = 32768
+
+    def oracle_rate(K, V, seconds):
+        t0, done = time.perf_counter(), 0
+        while time.perf_counter() - t0 < seconds or done == 0:
+            oq.quantize_keys(K)
+            oq.quantize_values(V)
+            done += K.shape[0]
+        return done * d * 2 * 2 / (time.perf_counter() - t0) / 1e9
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        rng = np.random.default_rng(3)
+        K = rng.standard_normal((sample_rows, d)).astype(np.float32)
+        V = rng.standard_normal((sample_rows, d)).astype(np.float32)
+        for _ in range(args.warmup):
+            oq.quantize_keys(K[:1024])
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oq.quantize_keys(K)
+            oq.quantize_values(V)
+        dt = (time.perf_counter() - t0) / args.steps
+        val = sample_rows * d * 2 * 2 / dt / 1e9
+        print(json.dumps({"metric": metric, "value": val, "unit": "GB/s", "impl": "reference", "n_gpus": 1,
+                          "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+                          "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                          "data": "synthetic", "config": cfg,
+                          "cpu_baseline": {"value": val, "unit": "GB/s", "cores": cpu_cores(), "kind": "oracle",
+                                           "sample": "%d rows of K and V per step" % sample_rows},
+                          "e2e": {"value": val, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}))
+        return
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(4)
+    K = torch.empty((rows, d), dtype=torch.bfloat16, device=dev).normal_(generator=gen)
+    V = torch.empty((rows, d), dtype=torch.bfloat16, device=dev).normal_(generator=gen)
+    out = vc.viscache_kv4_quantize(batch, prm, K, V)
+    hat = vc.viscache_kv4_dequantize(batch, prm, *out)
+
+    def quantize():
+        vc.viscache_kv4_quantize(batch, prm, K, V, out=out)
+
+    def dequantize():
+        vc.viscache_kv4_dequantize(batch, prm, *out, out=hat)
+
+    res = {}
+    clk = None
+    for name, fn in (("quantize", quantize), ("dequantize", dequantize)):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if name == "quantize":
+            clocks = ClockSampler(local)
+            clocks.start()
+        a.record()
+        for _ in range(args.steps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        if name == "quantize":
+            clk = clocks.stop()
+        vc.viscache_profile_enable(True)
+        for _ in range(args.steps):
+            fn()
+        torch.cuda.synchronize()
+        prof = vc.viscache_profile_read()
+        vc.viscache_profile_enable(False)
+        res[name] = (a.elapsed_time(b) / args.steps, {k: v[0] / args.steps for k, v in prof.items()},
+                     sum(v[1] for v in prof.values()))
+    ms, kern, launches = res["quantize"]
+    ms_dq, kern_dq, _ = res["dequantize"]
+    pk = peaks()
+    t_k = kern.get("kv4_quantize", float("nan")) * 1e-3
+    achieved = (in_bytes + out_bytes) / t_k / 1e9
+    # end to end: the cache from pinned host memory, codes and parameters back
+    hK, hV = K.cpu().pin_memory(), V.cpu().pin_memory()
+    dK, dV = torch.empty_like(K), torch.empty_like(V)
+    hout = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True) for x in out]
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        dK.copy_(hK, non_blocking=True)
+        dV.copy_(hV, non_blocking=True)
+        vc.viscache_kv4_quantize(batch, prm, dK, dV, out=out)
+        for h, x in zip(hout, out):
+            h.copy_(x, non_blocking=True)
+    b.record()
+    torch.cuda.synchronize()
+    ems = a.elapsed_time(b) / args.steps
+    Ks = K[:sample_rows].float().cpu().numpy()
+    Vs = V[:sample_rows].float().cpu().numpy()
+    cpu = oracle_rate(Ks, Vs, min(args.cpu_seconds, 5.0))
+    print(json.dumps({
+        "metric": metric, "value": in_bytes / (ms * 1e-3) / 1e9, "unit": "GB/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded normal cache)",
+        "config": dict(cfg, l2="%.2f GB of K and V per step > 129 MB L2" % (in_bytes / 1e9)),
+        "compression": in_bytes / out_bytes,
+        "dequantize": {"ms_per_step": ms_dq, "kernels_ms_per_step": kern_dq},
+        "kernels_ms_per_step": kern,
+        "roofline": {"kernel": "kv4_quantize", "bound": "hbm", "achieved": achieved, "peak": pk["hbm"],
+                     "unit": "GB/s", "frac": achieved / pk["hbm"], "traffic": None,
+                     "peak_source": pk["source"]},
+        "cpu_baseline": {"value": cpu, "unit": "GB/s", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": "%d rows of K and V, repeated for ~5 s (fp32 numpy)" % sample_rows},
+        "e2e": {"value": in_bytes / (ems * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": int(in_bytes),
+                "d2h_bytes_per_step": int(sum(x.numel() * x.element_size() for x in out))},
+        "gpu_launches": launches, "clocks": clk}))
+
+
 def main():
     args = parse()
+    if args.stage == "quant":
+        run_quant(args)
+        return
     if args.stage == "scout":
         run_scout(args)
         return

@@ -350,6 +350,43 @@ int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t
                               void* out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * viscache_kv4_* -- 4-bit quantisation of the compacted cache (Appendix
+ * "Quantization": the compressed visual KV combined with a 4-bit KV cache
+ * quantiser; the paper names KIVI-style quantisers without defining one).
+ * Asymmetric round-to-nearest with a per-group scale and minimum:
+ *     scale = (max - min) / 15,  code = clamp(rint((x - min) / scale), 0, 15)
+ *     (code 0 when scale = 0),   x_hat = code * scale + min (fused multiply-add),
+ * decided in fp32 (IEEE subtraction and division, rint to nearest even).
+ * Keys: per channel over groups of 32 consecutive rows of one (request,
+ * layer, KV head) segment of prunekv_compress's output (the last group of a
+ * segment may be shorter).  Values: per row over groups of 32 channels.
+ *
+ *   batch, p      the batch and parameters prunekv_compress ran with (d = 64
+ *                 or 128; bf16 or fp32 per p->dtype)
+ *   K_out, V_out  device [rows][d], prunekv_compress's outputs
+ *   K_codes, V_codes  device uint8 [rows][d/2]: two codes per byte, the even
+ *                 channel in the low nibble
+ *   K_params      device fp32 [key_groups][d][2]: (scale, min) per channel of
+ *                 each key group, groups in row order
+ *   V_params      device fp32 [rows][d/32][2]: (scale, min) per value group
+ *   K_hat, V_hat  device [rows][d] (dequantize): the reconstruction, rounded
+ *                 once to the input type
+ * viscache_kv4_sizes gives rows and key_groups for a batch (host only; either
+ * pointer may be NULL).  Float arrays 16-byte aligned.  All buffers are
+ * caller-owned; the calls are asynchronous on `stream` and need no workspace.
+ * Errors: VC_ERR_INVALID_ARG (shapes, NULL or misaligned pointers), the
+ * planner's errors for the batch, VC_ERR_CUDA.
+ */
+int viscache_kv4_sizes(const vc_batch* batch, const vc_params* p, int64_t* rows,
+                       int64_t* key_groups);
+int viscache_kv4_quantize(const vc_batch* batch, const vc_params* p, const void* K_out,
+                          const void* V_out, uint8_t* K_codes, uint8_t* V_codes, float* K_params,
+                          float* V_params, void* stream);
+int viscache_kv4_dequantize(const vc_batch* batch, const vc_params* p, const uint8_t* K_codes,
+                            const uint8_t* V_codes, const float* K_params, const float* V_params,
+                            void* K_hat, void* V_hat, void* stream);
+
+/*
  * Kernel path selection (process-wide, default VC_PATH_AUTO): AUTO runs the
  * score (Eq. token_score) and the fusion (Eq. redistribution, weight_fusion)
  * of bf16, d = 128 problems on the tcgen05 tensor cores and everything else

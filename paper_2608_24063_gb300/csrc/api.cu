@@ -459,6 +459,52 @@ DecodeWs decode_ws(int64_t units, int d, int pairs) {
   return w;
 }
 
+// The compacted cache's (request, layer) entries with B > 0, in row order,
+// cut into launches of at most kQuantMaxEntries entries.
+struct Kv4Plan {
+  std::vector<QuantTable> launches;   // tables (only .n entries used)
+  std::vector<int> units;             // key groups per launch
+  int64_t rows = 0, groups = 0;
+};
+int kv4_plan(const vc_params* p, const std::vector<RequestPlan>& plans, Kv4Plan* out) {
+  const int gr = kv4_group_rows();
+  out->launches.clear();
+  out->units.clear();
+  int64_t row = 0, groups = 0;
+  QuantTable cur;
+  cur.n = 0;
+  cur.pad = 0;
+  cur.unit_base = 0;
+  int units = 0;
+  auto flush = [&]() {
+    if (cur.n == 0) return;
+    out->launches.push_back(cur);
+    out->units.push_back(units);
+    cur.n = 0;
+    cur.unit_base = groups;
+    units = 0;
+  };
+  for (const RequestPlan& pl : plans) {
+    for (int l = 0; l < p->L; ++l) {
+      const int32_t b = pl.B[l];
+      if (b == 0) continue;
+      const int64_t u = (int64_t)p->Hkv * ((b + gr - 1) / gr);
+      if (cur.n == kQuantMaxEntries || units + u > (int64_t)1 << 30) flush();
+      QuantEntry& e = cur.e[cur.n++];
+      e.row0 = row;
+      e.B = b;
+      e.unit0 = units;
+      units += (int)u;
+      groups += u;
+      row += (int64_t)p->Hkv * b;
+    }
+  }
+  flush();
+  out->rows = row;
+  out->groups = groups;
+  return VC_OK;
+}
+
 }  // namespace
 }  // namespace vc
 
@@ -649,6 +695,52 @@ int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t
                                    reinterpret_cast<float2*>(w + dw.o_ml),
                                    reinterpret_cast<int32_t*>(w + dw.o_arr),
                                    static_cast<cudaStream_t>(stream)));
+}
+
+int viscache_kv4_sizes(const vc_batch* batch, const vc_params* p, int64_t* rows, int64_t* key_groups) {
+  std::vector<RequestPlan> plans;
+  const int rc = plan_batch(batch, p, &plans);
+  if (rc != VC_OK) return rc;
+  Kv4Plan kp;
+  kv4_plan(p, plans, &kp);
+  if (rows) *rows = kp.rows;
+  if (key_groups) *key_groups = kp.groups;
+  return VC_OK;
+}
+
+static int kv4_run(const vc_batch* batch, const vc_params* p, bool quantize, const void* K,
+                   const void* V, uint8_t* Kc, uint8_t* Vc, float* Kp, float* Vp, void* Kh, void* Vh,
+                   void* stream) {
+  std::vector<RequestPlan> plans;
+  const int rc = plan_batch(batch, p, &plans);
+  if (rc != VC_OK) return rc;
+  if (!Kc || !Vc || !Kp || !Vp || !aligned16(Kp) || !aligned16(Vp)) return VC_ERR_INVALID_ARG;
+  if (quantize ? (!K || !V || !aligned16(K) || !aligned16(V)) : (!Kh || !Vh || !aligned16(Kh) || !aligned16(Vh)))
+    return VC_ERR_INVALID_ARG;
+  static thread_local Kv4Plan kp;
+  kv4_plan(p, plans, &kp);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  for (size_t i = 0; i < kp.launches.size(); ++i) {
+    const cudaError_t e = launch_kv4(kp.launches[i], kp.units[i], p->dtype, p->d, quantize, K, V, Kc,
+                                     Vc, Kp, Vp, Kh, Vh, st);
+    if (e != cudaSuccess) return VC_ERR_CUDA;
+  }
+  return VC_OK;
+}
+
+int viscache_kv4_quantize(const vc_batch* batch, const vc_params* p, const void* K_out,
+                          const void* V_out, uint8_t* K_codes, uint8_t* V_codes, float* K_params,
+                          float* V_params, void* stream) {
+  return kv4_run(batch, p, true, K_out, V_out, K_codes, V_codes, K_params, V_params, nullptr, nullptr,
+                 stream);
+}
+
+int viscache_kv4_dequantize(const vc_batch* batch, const vc_params* p, const uint8_t* K_codes,
+                            const uint8_t* V_codes, const float* K_params, const float* V_params,
+                            void* K_hat, void* V_hat, void* stream) {
+  return kv4_run(batch, p, false, nullptr, nullptr, const_cast<uint8_t*>(K_codes),
+                 const_cast<uint8_t*>(V_codes), const_cast<float*>(K_params),
+                 const_cast<float*>(V_params), K_hat, V_hat, stream);
 }
 
 }  // extern "C"

@@ -91,4 +91,24 @@ cudaError_t launch_decode(const DecodeTable& tb, int dtype, int d, const void* q
                           const void* Vc, const void* Kt, const void* Vt, void* out, float* part_o,
                           float2* part_ml, int32_t* arrivals, cudaStream_t st);
 
+// 4-bit quantisation of the compacted cache: per (request, layer) with B > 0,
+// Hkv segments of B rows starting at row0 (KV head g at row0 + g * B); a
+// unit is one group of up to kv4_group_rows() rows of one segment.
+struct QuantEntry {
+  int64_t row0;            // first row of the (request, layer)
+  int32_t B;               // rows per KV head
+  int32_t unit0;           // first unit of the entry within the launch
+};
+constexpr int kQuantMaxEntries = 1792;
+struct QuantTable {
+  int32_t n;               // entries
+  int32_t pad;
+  int64_t unit_base;       // global index of the launch's first key group
+  QuantEntry e[kQuantMaxEntries];
+};
+int kv4_group_rows();
+cudaError_t launch_kv4(const QuantTable& tb, int units, int dtype, int d, bool quantize,
+                       const void* K, const void* V, uint8_t* Kc, uint8_t* Vc, float* Kp, float* Vp,
+                       void* Kh, void* Vh, cudaStream_t st);
+
 }  // namespace vc

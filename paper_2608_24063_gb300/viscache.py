@@ -40,7 +40,8 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
             "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
             "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr",
-            "viscache_decode_workspace_size", "viscache_decode_attention")
+            "viscache_decode_workspace_size", "viscache_decode_attention",
+            "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize")
 
 
 class VisCacheError(RuntimeError):
@@ -81,6 +82,12 @@ def lib() -> ctypes.CDLL:
         L.viscache_scout_workspace_size.argtypes = [i32, pi32, i32]
         L.viscache_scout_workspace_size.restype = sz
         L.viscache_scout_mmr.argtypes = [vp, vp, i32, pi32, i32, f32, u32, u32, vp, vp, vp, pi32, vp, sz, vp]
+        L.viscache_kv4_sizes.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params),
+                                         ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+        L.viscache_kv4_quantize.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), vp, vp,
+                                            vp, vp, vp, vp, vp]
+        L.viscache_kv4_dequantize.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), vp, vp,
+                                              vp, vp, vp, vp, vp]
         L.viscache_decode_workspace_size.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), pi32]
         L.viscache_decode_workspace_size.restype = sz
         L.viscache_decode_attention.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), i32,
@@ -392,6 +399,47 @@ def viscache_decode_attention(batch: Batch, params: vc_params, layer: int, q: to
         ctypes.byref(batch.c), ctypes.byref(params), int(layer), _ptr(q), _ptr(K_out), _ptr(V_out),
         _ptr(K_text), _ptr(V_text), nt, _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
     return out
+
+
+def viscache_kv4_sizes(batch: Batch, params: vc_params) -> Tuple[int, int]:
+    """(rows, key groups) of the compacted cache's 4-bit form."""
+    rows, groups = ctypes.c_int64(0), ctypes.c_int64(0)
+    _check("viscache_kv4_sizes", lib().viscache_kv4_sizes(ctypes.byref(batch.c), ctypes.byref(params),
+                                                          ctypes.byref(rows), ctypes.byref(groups)))
+    return rows.value, groups.value
+
+
+def viscache_kv4_quantize(batch: Batch, params: vc_params, K_out: torch.Tensor, V_out: torch.Tensor,
+                          out=None, stream=None):
+    """4-bit codes and (scale, min) parameters of the compacted cache:
+    returns (K_codes [rows][d/2], V_codes [rows][d/2], K_params [groups][d][2], V_params [rows][d/32][2])."""
+    rows, groups = viscache_kv4_sizes(batch, params)
+    d, dev = params.d, K_out.device
+    if out is None:
+        out = (torch.empty((max(rows, 1), d // 2), dtype=torch.uint8, device=dev),
+               torch.empty((max(rows, 1), d // 2), dtype=torch.uint8, device=dev),
+               torch.empty((max(groups, 1), d, 2), dtype=torch.float32, device=dev),
+               torch.empty((max(rows, 1), d // 32, 2), dtype=torch.float32, device=dev))
+    kc, vc_, kp, vp_ = out
+    _check("viscache_kv4_quantize", lib().viscache_kv4_quantize(
+        ctypes.byref(batch.c), ctypes.byref(params), _ptr(K_out), _ptr(V_out), _ptr(kc), _ptr(vc_),
+        _ptr(kp), _ptr(vp_), _stream(stream)))
+    return kc[:rows], vc_[:rows], kp[:groups], vp_[:rows]
+
+
+def viscache_kv4_dequantize(batch: Batch, params: vc_params, K_codes: torch.Tensor, V_codes: torch.Tensor,
+                            K_params: torch.Tensor, V_params: torch.Tensor, dtype=torch.bfloat16,
+                            out=None, stream=None):
+    """Reconstruction (K_hat, V_hat) [rows][d] of the 4-bit cache in `dtype`."""
+    rows = K_codes.shape[0]
+    if out is None:
+        out = (torch.empty((max(rows, 1), params.d), dtype=dtype, device=K_codes.device),
+               torch.empty((max(rows, 1), params.d), dtype=dtype, device=K_codes.device))
+    kh, vh = out
+    _check("viscache_kv4_dequantize", lib().viscache_kv4_dequantize(
+        ctypes.byref(batch.c), ctypes.byref(params), _ptr(K_codes), _ptr(V_codes), _ptr(K_params),
+        _ptr(V_params), _ptr(kh), _ptr(vh), _stream(stream)))
+    return kh[:rows], vh[:rows]
 
 
 def viscache_set_kernel_path(path: int) -> None:

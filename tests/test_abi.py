@@ -168,3 +168,28 @@ def test_decode_workspace_covers_every_layer():
     assert got % 256 == 0 and got >= units * 8 * (128 * 4 + 8)
     assert vc.viscache_decode_workspace_size(b, prm) <= got
     assert vc.viscache_decode_workspace_size(vc.Batch([100] * 257, [8] * 257, [(1, 4)] * 257), prm) == 0
+
+
+def test_kv4_sizes_match_the_oracle_layout():
+    from oracle import quant as oq
+    ns, rrs, L, Hkv = [12544, 700, 33], [(19, 100), (25, 100), (50, 100)], 28, 4
+    b = vc.Batch(ns, [64] * 3, rrs)
+    prm = vc.make_params(L, 28, Hkv, 128, vc.VC_BF16)
+    Bs = [plan.plan_budgets(L, n, Fraction(*rr))[0] for n, rr in zip(ns, rrs)]
+    rows, groups = vc.viscache_kv4_sizes(b, prm)
+    segs = oq.segments(Bs, Hkv)
+    assert rows == sum(n for _, n in segs)
+    assert groups == sum(-(-n // oq.GROUP) for _, n in segs)
+
+
+def test_kv4_entries_reject_bad_arguments_without_touching_the_device():
+    lib = vc.lib()
+    p = ctypes.c_void_p(256)
+    b = vc.Batch([100], [8], [(25, 100)])
+    prm = vc.make_params(4, 8, 2, 128, vc.VC_BF16)
+    args = lambda *x: (ctypes.byref(b.c), ctypes.byref(prm)) + x
+    assert lib.viscache_kv4_quantize(*args(p, p, None, p, p, p, None)) == vc.VC_ERR_INVALID_ARG
+    assert lib.viscache_kv4_quantize(*args(p, p, p, p, ctypes.c_void_p(260), p, None)) == vc.VC_ERR_INVALID_ARG
+    assert lib.viscache_kv4_dequantize(*args(p, p, p, p, None, p, None)) == vc.VC_ERR_INVALID_ARG
+    bad = vc.make_params(4, 8, 2, 96, vc.VC_BF16)
+    assert lib.viscache_kv4_sizes(ctypes.byref(b.c), ctypes.byref(bad), None, None) == vc.VC_ERR_INVALID_ARG

@@ -49,7 +49,7 @@ def parse():
     ap.add_argument("--stage", choices=["prunekv", "scout", "decode", "quant"], default="prunekv",
                     help="prunekv: the compression pass (the headline); scout: MMR keyframe selection")
     ap.add_argument("--requests", type=int, default=16, help="--stage decode: concurrent requests")
-    ap.add_argument("--decode-cache", choices=["both", "compressed", "full"], default="both",
+    ap.add_argument("--decode-cache", choices=["both", "compressed", "full", "kv4"], default="both",
                     help="--stage decode: which caches to time")
     ap.add_argument("--rank", choices=["shared", "per_layer"], default="shared",
                     help="ranking: one order per KV head from the layer mean (method default) or per layer")
@@ -439,10 +439,14 @@ def run_decode(args):
     prm_f = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16, h=L, m=(1, 1), schedule=vc.VC_SCHED_FIXED)
     rows_c = vc.compressed_rows(batch_c, prm_c)
     texts = [T] * n_req
-    names = ("full", "compressed") if args.decode_cache == "both" else (args.decode_cache,)
+    names = ("full", "compressed", "kv4") if args.decode_cache == "both" else (args.decode_cache,)
     caches = {}
-    if "compressed" in names:
+    if "compressed" in names or "kv4" in names:
         caches["compressed"] = (batch_c, prm_c, normal(rows_c, d), normal(rows_c, d))
+    if "kv4" in names:
+        # the compressed cache's visual rows in 4-bit form
+        kv4 = vc.viscache_kv4_quantize(batch_c, prm_c, caches["compressed"][2], caches["compressed"][3])
+        caches["kv4"] = (batch_c, prm_c, kv4, None)
     if "full" in names:
         caches["full"] = (batch_f, prm_f, normal(n_req * L * Hkv * n, d), normal(n_req * L * Hkv * n, d))
     Kt, Vt = normal(L, n_req * Hkv * T, d), normal(L, n_req * Hkv * T, d)
@@ -450,11 +454,16 @@ def run_decode(args):
     out = torch.empty_like(q)
     ws = torch.empty(max(vc.viscache_decode_workspace_size(b, p, texts) for b, p, _, _ in caches.values()),
                      dtype=torch.uint8, device=dev)
+    if args.decode_cache == "kv4":
+        del caches["compressed"]
 
     def step(name, qq=q):
         b, p, K, V = caches[name]
         for l in range(L):
-            vc.viscache_decode_attention(b, p, l, qq[l], K, V, Kt[l], Vt[l], texts, out=out[l], ws=ws)
+            if name == "kv4":
+                vc.viscache_decode_attention_kv4(b, p, l, qq[l], K, Kt[l], Vt[l], texts, out=out[l], ws=ws)
+            else:
+                vc.viscache_decode_attention(b, p, l, qq[l], K, V, Kt[l], Vt[l], texts, out=out[l], ws=ws)
 
     res = {}
     clk = None
@@ -499,10 +508,16 @@ def run_decode(args):
         # one cache alone (a profiling run): its time and kernel split only
         ms, kern, launches = res[names[0]]
         print(json.dumps({"stage": "decode", "cache": names[0], "requests": n_req, "ms_per_step": ms,
-                          "kernels_ms_per_step": kern, "launches_per_step": launches, "clocks": clk}))
+                          "kv4_cache": {"ms_per_step": ms_q4, "value": n_req / (ms_q4 * 1e-3),
+                      "speedup_vs_compressed": ms / ms_q4, "kernels_ms_per_step": kern_q4,
+                      "cache_bytes_per_step": int(sum(n_req * Hkv * b for b in B) * (d + d // 32 * 8)
+                                                  + sum(n_req * Hkv * -(-b // 32) * d * 8 for b in B)
+                                                  + L * n_req * Hkv * T * d * 2 * 2)},
+        "kernels_ms_per_step": kern, "launches_per_step": launches, "clocks": clk}))
         return
     ms, kern, launches = res["compressed"]
     ms_full, kern_full, _ = res["full"]
+    ms_q4, kern_q4, _ = res["kv4"]
     # algorithmic bytes of a step: every cached K and V row of every layer once
     # plus the query rows (the main kernel, L launches a step); achieved =
     # those bytes over the launches' summed event time
@@ -559,6 +574,11 @@ def run_decode(args):
                        "speedup_of_compressed": ms_full / ms,
                        "kernels_ms_per_step": kern_full,
                        "main_kernel_gbs": achieved_f},
+        "kv4_cache": {"ms_per_step": ms_q4, "value": n_req / (ms_q4 * 1e-3),
+                      "speedup_vs_compressed": ms / ms_q4, "kernels_ms_per_step": kern_q4,
+                      "cache_bytes_per_step": int(sum(n_req * Hkv * b for b in B) * (d + d // 32 * 8)
+                                                  + sum(n_req * Hkv * -(-b // 32) * d * 8 for b in B)
+                                                  + L * n_req * Hkv * T * d * 2 * 2)},
         "kernels_ms_per_step": kern,
         "roofline": {"kernel": main_kernel, "bound": "hbm", "achieved": achieved,
                      "peak": pk["hbm"], "unit": "GB/s", "frac": achieved / pk["hbm"], "traffic": None,

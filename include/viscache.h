@@ -344,6 +344,19 @@ int viscache_profile_read(char* names, int name_bytes, float* total_ms, int* lau
  */
 size_t viscache_decode_workspace_size(const vc_batch* batch, const vc_params* p,
                                       const int32_t* n_text);
+/*
+ * viscache_decode_attention_kv4 -- the same step over the 4-bit form of the
+ * visual rows (viscache_kv4_quantize's outputs for the same batch and
+ * parameters; bf16 only): each visual row is expanded to code * scale + min
+ * rounded to bf16, exactly the rows viscache_kv4_dequantize writes, and the
+ * attention is then the one above.  Text rows, queries and output are bf16;
+ * the workspace is viscache_decode_workspace_size's.  Errors as above.
+ */
+int viscache_decode_attention_kv4(const vc_batch* batch, const vc_params* p, int32_t layer,
+                                  const void* q, const uint8_t* K_codes, const uint8_t* V_codes,
+                                  const float* K_params, const float* V_params, const void* K_text,
+                                  const void* V_text, const int32_t* n_text, void* out, void* ws,
+                                  size_t ws_bytes, void* stream);
 int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t layer,
                               const void* q, const void* K_out, const void* V_out,
                               const void* K_text, const void* V_text, const int32_t* n_text,

@@ -420,16 +420,27 @@ int decode_table(const vc_params* p, const std::vector<RequestPlan>& plans, int 
   }
   const int split = decode_split_keys(p->dtype);
   tb->split = split;
-  int64_t rows = 0, text = 0, units = 0;
+  int64_t rows = 0, text = 0, units = 0, kgroups = 0;
+  const int gr = kv4_group_rows();
   for (int r = 0; r < n_req; ++r) {
     const RequestPlan& pl = plans[r];
     const int32_t T = n_text ? n_text[r] : 0;
-    int64_t P = 0, all = 0;
+    int64_t P = 0, all = 0, KG = 0, allg = 0;
     for (int l = 0; l < p->L; ++l) {
-      if (l < layer) P += pl.B[l];
+      const int64_t g = (pl.B[l] + gr - 1) / gr;
+      if (l < layer) {
+        P += pl.B[l];
+        KG += g;
+      }
       all += pl.B[l];
+      allg += g;
     }
     DecodeReq& q = tb->req[r];
+    // key groups of the 4-bit form are stacked in row order: request, layer, KV head
+    q.kg0 = kgroups + (int64_t)p->Hkv * KG;
+    q.nkg = (int32_t)((pl.B[layer] + gr - 1) / gr);
+    q.pad = 0;
+    kgroups += (int64_t)p->Hkv * allg;
     q.vis_row0 = rows + (int64_t)p->Hkv * P;
     q.txt_row0 = text;
     q.B = pl.B[layer];
@@ -695,6 +706,35 @@ int viscache_decode_attention(const vc_batch* batch, const vc_params* p, int32_t
                                    reinterpret_cast<float2*>(w + dw.o_ml),
                                    reinterpret_cast<int32_t*>(w + dw.o_arr),
                                    static_cast<cudaStream_t>(stream)));
+}
+
+int viscache_decode_attention_kv4(const vc_batch* batch, const vc_params* p, int32_t layer,
+                                  const void* q, const uint8_t* K_codes, const uint8_t* V_codes,
+                                  const float* K_params, const float* V_params, const void* K_text,
+                                  const void* V_text, const int32_t* n_text, void* out, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  std::vector<RequestPlan> plans;
+  const int rc = plan_batch(batch, p, &plans);
+  if (rc != VC_OK) return rc;
+  if (p->dtype != VC_BF16 || layer < 0 || layer >= p->L) return VC_ERR_INVALID_ARG;
+  if (!q || !K_codes || !V_codes || !K_params || !V_params || !out || !aligned16(q) ||
+      !aligned16(K_codes) || !aligned16(V_codes) || !aligned16(K_params) || !aligned16(V_params) ||
+      !aligned16(out))
+    return VC_ERR_INVALID_ARG;
+  if (n_text && (!K_text || !V_text || !aligned16(K_text) || !aligned16(V_text)))
+    return VC_ERR_INVALID_ARG;
+  static thread_local DecodeTable tb;
+  const int tc = decode_table(p, plans, layer, n_text, &tb);
+  if (tc != VC_OK) return tc;
+  const DecodeWs dw = decode_ws(tb.units, p->d, tb.n_req * tb.Hkv);
+  const int wc = check_ws(ws, ws_bytes, dw.total);
+  if (wc != VC_OK) return wc;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  return cuda_status(launch_decode_kv4(tb, p->d, q, K_codes, V_codes, K_params, V_params, K_text,
+                                       V_text, out, reinterpret_cast<float*>(w + dw.o_o),
+                                       reinterpret_cast<float2*>(w + dw.o_ml),
+                                       reinterpret_cast<int32_t*>(w + dw.o_arr),
+                                       static_cast<cudaStream_t>(stream)));
 }
 
 int viscache_kv4_sizes(const vc_batch* batch, const vc_params* p, int64_t* rows, int64_t* key_groups) {

@@ -8,14 +8,16 @@
 // of the keys); a split's rows are staged in shared memory by 16-byte
 // asynchronous copies (the whole split in flight at once), the row's 16-byte
 // pieces XOR-permuted so that the reads hit distinct banks.
-//   decode_mma_kernel      (bf16 caches, splits of 128 keys) K and V rows in
-//                          two buffers, loaded together; QK^T and PV as
-//                          mma.sync m16n8k16 tiles: keys, then output
-//                          dimensions, as M and the G <= 8 query heads as
-//                          N = 8; the split's softmax in between.  The CTA
-//                          that finishes the last split of a (request, KV
-//                          head) merges the pair's split states into the
-//                          output.
+//   decode_mma_kernel      (bf16 caches, splits of 256 keys) K rows, then V
+//                          rows, in one buffer; QK^T and PV as mma.sync
+//                          m16n8k16 tiles: keys, then output dimensions, as
+//                          M and the G <= 8 query heads as N = 8; the
+//                          split's softmax in between.  The CTA that
+//                          finishes the last split of a (request, KV head)
+//                          merges the pair's split states into the output.
+//                          Its Q4 form reads the visual rows from the 4-bit
+//                          cache (codes and parameters loaded into registers
+//                          and expanded to bf16 rows in the same buffer).
 //   decode_partial_kernel  (fp32 caches, splits of 256 keys) the same steps on
 //                          CUDA cores, K then V rows in one buffer: two
 //                          threads per key pair form the logits with packed
@@ -320,6 +322,7 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], 
 struct UnitRows {
   int r, g, nk, nv, pair, nsplit;
   int64_t vis0, txt0, u_first;   // first visual / text row, first unit of the (request, KV head)
+  int64_t kg;                    // 4-bit cache: the split's first key group
 };
 __device__ __forceinline__ UnitRows unit_rows(const DecodeTable& tb, int unit) {
   UnitRows x;
@@ -336,6 +339,7 @@ __device__ __forceinline__ UnitRows unit_rows(const DecodeTable& tb, int unit) {
   x.pair = x.r * tb.Hkv + x.g;
   x.nsplit = rq.nsplit;
   x.u_first = rq.unit0 + (int64_t)x.g * rq.nsplit;
+  x.kg = rq.kg0 + (int64_t)x.g * rq.nkg + k0 / 32;
   return x;
 }
 
@@ -348,14 +352,16 @@ __device__ __forceinline__ UnitRows unit_rows(const DecodeTable& tb, int unit) {
 template <int D>
 __device__ __forceinline__ void stage_split(uint32_t buf_s, const __nv_bfloat16* vis,
                                             const __nv_bfloat16* txt, int nv, int nk,
-                                            const __nv_bfloat16* zsrc) {
+                                            const __nv_bfloat16* zsrc, int first = 0) {
   using C = MmaCfg<D>;
   constexpr int RSTEP = kDecThreads / C::PR;
   static_assert(RSTEP % 8 == 0, "row step keeps the XOR slot");
   const int c = (int)threadIdx.x % C::PR, r0 = (int)threadIdx.x / C::PR;
   const int rows = min(kSplitM, (nk + 15) & ~15);
   const uint32_t dst0 = buf_s + r0 * C::RB + mma_slot(r0, c) * 16;
-  for (int r = r0; r < rows; r += RSTEP) {
+  int r = r0;                                   // first row >= `first` in this thread's column
+  if (first > r0) r += (first - r0 + RSTEP - 1) / RSTEP * RSTEP;
+  for (; r < rows; r += RSTEP) {
     const __nv_bfloat16* src = r < nv ? vis + (int64_t)r * D + c * 8
                              : r < nk ? txt + (int64_t)(r - nv) * D + c * 8 : zsrc;
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst0 + (r - r0) * C::RB),
@@ -374,19 +380,76 @@ __device__ __forceinline__ void stage_q(uint32_t qbuf_s, const __nv_bfloat16* qr
   }
 }
 
+// 4-bit visual rows [0, nv) of a split expanded into bf16 rows of the
+// (XOR-permuted) row buffer: x = fma(code, scale, min) rounded to bf16, the
+// rows viscache_kv4_dequantize writes.  Thread t owns the 8-channel piece
+// c = t % PR of the PR consecutive rows (t / PR) * PR ...; those rows lie in
+// one 32-row key group, so a key thread loads its 8 channels' parameters
+// once.  Codes: D/2 bytes a row (4 bytes per piece); KEYS: parameters per
+// (key group, channel) from `par` (the split's first group); values: per
+// (row, 32-channel group) from `par` (the split's first row).
+template <int D, bool KEYS>
+__device__ __forceinline__ void expand_q4(uint8_t* buf, const uint8_t* codes, const float* par, int nv) {
+  using C = MmaCfg<D>;
+  constexpr int RPT = kSplitM * C::PR / kDecThreads;   // rows per thread (= PR)
+  static_assert(32 % RPT == 0, "a thread's rows lie in one key group");
+  const int c = (int)threadIdx.x % C::PR, r0 = (int)threadIdx.x / C::PR * RPT;
+  if (r0 >= nv) return;
+  uint32_t w[RPT];
+#pragma unroll
+  for (int i = 0; i < RPT; ++i)
+    w[i] = r0 + i < nv ? *reinterpret_cast<const uint32_t*>(codes + (size_t)(r0 + i) * (D / 2) + 4 * c) : 0u;
+  if (KEYS) {
+    float4 pk[4];                                 // (scale, min) of channels 8c + 2j, 8c + 2j + 1
+    const float4* pp = reinterpret_cast<const float4*>(par + ((size_t)(r0 >> 5) * D + 8 * c) * 2);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) pk[j] = pp[j];
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) {
+      if (r0 + i >= nv) break;
+      float x[8];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        x[2 * j] = fmaf((float)((w[i] >> (8 * j)) & 15u), pk[j].x, pk[j].y);
+        x[2 * j + 1] = fmaf((float)((w[i] >> (8 * j + 4)) & 15u), pk[j].z, pk[j].w);
+      }
+      const int r = r0 + i;
+      *reinterpret_cast<uint4*>(buf + (size_t)r * C::RB + mma_slot(r, c) * 16) =
+          make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+    }
+  } else {
+    float2 pv[RPT];
+#pragma unroll
+    for (int i = 0; i < RPT; ++i)
+      pv[i] = r0 + i < nv ? reinterpret_cast<const float2*>(par)[(size_t)(r0 + i) * (D / 32) + (c >> 2)]
+                          : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) {
+      if (r0 + i >= nv) break;
+      float x[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[j] = fmaf((float)((w[i] >> (4 * j)) & 15u), pv[i].x, pv[i].y);
+      const int r = r0 + i;
+      *reinterpret_cast<uint4*>(buf + (size_t)r * C::RB + mma_slot(r, c) * 16) =
+          make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+    }
+  }
+}
+
 // Decode kernel for bf16 caches: one CTA per unit (request, KV head, split
 // of kSplitM keys), three CTAs per SM.  The split's K rows (with the query
 // rows) load first; its V rows load into the same buffer during the softmax.
 // The CTA that completes the last split of a (request, KV head) merges that
 // pair's split states into `out`: an arrival count per pair; no CTA ever
 // waits for another.
-template <int D>
+template <int D, bool Q4>
 __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     const __grid_constant__ DecodeTable tb, const __nv_bfloat16* __restrict__ q,
     const __nv_bfloat16* __restrict__ Kc, const __nv_bfloat16* __restrict__ Vc,
     const __nv_bfloat16* __restrict__ Kt, const __nv_bfloat16* __restrict__ Vt,
-    float* __restrict__ part_o, float2* __restrict__ part_ml, int32_t* __restrict__ arrivals,
-    __nv_bfloat16* __restrict__ out) {
+    const uint8_t* __restrict__ Kq, const uint8_t* __restrict__ Vq, const float* __restrict__ Kqp,
+    const float* __restrict__ Vqp, float* __restrict__ part_o, float2* __restrict__ part_ml,
+    int32_t* __restrict__ arrivals, __nv_bfloat16* __restrict__ out) {
   using C = MmaCfg<D>;
   extern __shared__ __align__(128) uint8_t dsm[];
   uint8_t* buf = dsm;                           // K rows, V rows, warp partials, merge weights
@@ -406,9 +469,11 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   const int unit = blockIdx.x;
   const UnitRows cur = unit_rows(tb, unit);
   const int nk = cur.nk;
-  stage_split<D>(buf_s, Kc + cur.vis0 * D, Kt + cur.txt0 * D, cur.nv, nk, q);
+  if (Q4) stage_split<D>(buf_s, Kc, Kt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
+  else stage_split<D>(buf_s, Kc + cur.vis0 * D, Kt + cur.txt0 * D, cur.nv, nk, q);
   stage_q<D>(qbuf_s, q + ((int64_t)cur.r * tb.Hq + cur.g * G) * D, G);
   tc::cp_async_commit();
+  if (Q4) expand_q4<D, true>(buf, Kq + cur.vis0 * (D / 2), Kqp + cur.kg * D * 2, cur.nv);
   tc::cp_async_wait<0>();
   __syncthreads();
   // B fragments of Q^T (k = dimension, n = query) in log2 units, high + low,
@@ -454,8 +519,14 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     }
   }
   __syncthreads();                              // K rows, query rows, fragments read: stage V
-  stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q);
-  tc::cp_async_commit();
+  if (Q4) {
+    stage_split<D>(buf_s, Vc, Vt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
+    tc::cp_async_commit();
+    expand_q4<D, false>(buf, Vq + cur.vis0 * (D / 2), Vqp + cur.vis0 * (D / 32) * 2, cur.nv);
+  } else {
+    stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q);
+    tc::cp_async_commit();
+  }
   // softmax over the split: lane holds keys (16 mt + gid, + 8) x queries (2 tig, + 1)
   float x[C::TPW][4];
   float m0 = -INFINITY, m1 = -INFINITY;
@@ -748,30 +819,31 @@ cudaError_t launch_decode_t(const DecodeTable& tb, const void* q, const void* Kc
   return cudaGetLastError();
 }
 
-template <int D>
+template <int D, bool Q4>
 cudaError_t launch_decode_mma(const DecodeTable& tb, const void* q, const void* Kc, const void* Vc,
-                              const void* Kt, const void* Vt, void* out, float* part_o,
+                              const void* Kt, const void* Vt, const uint8_t* Kq, const uint8_t* Vq,
+                              const float* Kqp, const float* Vqp, void* out, float* part_o,
                               float2* part_ml, int32_t* arrivals, cudaStream_t st) {
   using B16 = __nv_bfloat16;
   if (tb.units < 1) return cudaSuccess;
   constexpr size_t smem = MmaCfg<D>::SMEM;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(decode_mma_kernel<D>,
+    cudaError_t e = cudaFuncSetAttribute(decode_mma_kernel<D, Q4>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     // the whole unified L1 as shared memory: three CTAs per SM
-    e = cudaFuncSetAttribute(decode_mma_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    e = cudaFuncSetAttribute(decode_mma_kernel<D, Q4>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   cudaError_t e = cudaMemsetAsync(arrivals, 0, sizeof(int32_t) * tb.n_req * tb.Hkv, st);
   if (e != cudaSuccess) return e;
-  ProfileScope ps("decode_attn", st);
-  decode_mma_kernel<D><<<(unsigned)tb.units, kDecThreads, smem, st>>>(
+  ProfileScope ps(Q4 ? "decode_attn_kv4" : "decode_attn", st);
+  decode_mma_kernel<D, Q4><<<(unsigned)tb.units, kDecThreads, smem, st>>>(
       tb, static_cast<const B16*>(q), static_cast<const B16*>(Kc), static_cast<const B16*>(Vc),
-      static_cast<const B16*>(Kt), static_cast<const B16*>(Vt), part_o, part_ml, arrivals,
-      static_cast<B16*>(out));
+      static_cast<const B16*>(Kt), static_cast<const B16*>(Vt), Kq, Vq, Kqp, Vqp, part_o, part_ml,
+      arrivals, static_cast<B16*>(out));
   return cudaGetLastError();
 }
 
@@ -783,11 +855,25 @@ cudaError_t launch_decode(const DecodeTable& tb, int dtype, int d, const void* q
                           const void* Vc, const void* Kt, const void* Vt, void* out, float* part_o,
                           float2* part_ml, int32_t* arrivals, cudaStream_t st) {
   if (dtype == VC_BF16) {
-    if (d == 128) return launch_decode_mma<128>(tb, q, Kc, Vc, Kt, Vt, out, part_o, part_ml, arrivals, st);
-    return launch_decode_mma<64>(tb, q, Kc, Vc, Kt, Vt, out, part_o, part_ml, arrivals, st);
+    if (d == 128)
+      return launch_decode_mma<128, false>(tb, q, Kc, Vc, Kt, Vt, nullptr, nullptr, nullptr, nullptr, out,
+                                           part_o, part_ml, arrivals, st);
+    return launch_decode_mma<64, false>(tb, q, Kc, Vc, Kt, Vt, nullptr, nullptr, nullptr, nullptr, out,
+                                        part_o, part_ml, arrivals, st);
   }
   if (d == 128) return launch_decode_t<float, 128>(tb, q, Kc, Vc, Kt, Vt, out, part_o, part_ml, st);
   return launch_decode_t<float, 64>(tb, q, Kc, Vc, Kt, Vt, out, part_o, part_ml, st);
+}
+
+cudaError_t launch_decode_kv4(const DecodeTable& tb, int d, const void* q, const uint8_t* Kq,
+                              const uint8_t* Vq, const float* Kqp, const float* Vqp, const void* Kt,
+                              const void* Vt, void* out, float* part_o, float2* part_ml,
+                              int32_t* arrivals, cudaStream_t st) {
+  if (d == 128)
+    return launch_decode_mma<128, true>(tb, q, nullptr, nullptr, Kt, Vt, Kq, Vq, Kqp, Vqp, out, part_o,
+                                        part_ml, arrivals, st);
+  return launch_decode_mma<64, true>(tb, q, nullptr, nullptr, Kt, Vt, Kq, Vq, Kqp, Vqp, out, part_o,
+                                     part_ml, arrivals, st);
 }
 
 }  // namespace vc

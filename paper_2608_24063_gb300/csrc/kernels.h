@@ -78,6 +78,9 @@ struct DecodeReq {
   int32_t B, T;            // visual and text rows per KV head
   int32_t unit0;           // first (KV head, split) unit of the request
   int32_t nsplit;          // splits per KV head, max(1, ceil((B+T) / split keys))
+  int64_t kg0;             // 4-bit cache: first key group of KV head 0 in this layer
+  int32_t nkg;             // 4-bit cache: key groups per KV head, ceil(B / 32)
+  int32_t pad;
 };
 struct DecodeTable {
   int32_t n_req, Hq, Hkv, G;
@@ -87,6 +90,12 @@ struct DecodeTable {
   DecodeReq req[kDecodeMaxReq];
 };
 int decode_split_keys(int dtype);   // the largest split a kernel takes
+// Decode over the 4-bit form of the visual rows (viscache_kv4_quantize's
+// codes and parameters; bf16 query, text rows and output).
+cudaError_t launch_decode_kv4(const DecodeTable& tb, int d, const void* q, const uint8_t* Kq,
+                              const uint8_t* Vq, const float* Kqp, const float* Vqp, const void* Kt,
+                              const void* Vt, void* out, float* part_o, float2* part_ml,
+                              int32_t* arrivals, cudaStream_t st);
 cudaError_t launch_decode(const DecodeTable& tb, int dtype, int d, const void* q, const void* Kc,
                           const void* Vc, const void* Kt, const void* Vt, void* out, float* part_o,
                           float2* part_ml, int32_t* arrivals, cudaStream_t st);

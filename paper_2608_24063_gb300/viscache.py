@@ -41,7 +41,8 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
             "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr",
             "viscache_decode_workspace_size", "viscache_decode_attention",
-            "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize")
+            "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize",
+            "viscache_decode_attention_kv4")
 
 
 class VisCacheError(RuntimeError):
@@ -88,6 +89,8 @@ def lib() -> ctypes.CDLL:
                                             vp, vp, vp, vp, vp]
         L.viscache_kv4_dequantize.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), vp, vp,
                                               vp, vp, vp, vp, vp]
+        L.viscache_decode_attention_kv4.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), i32,
+                                                    vp, vp, vp, vp, vp, vp, vp, pi32, vp, vp, sz, vp]
         L.viscache_decode_workspace_size.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), pi32]
         L.viscache_decode_workspace_size.restype = sz
         L.viscache_decode_attention.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params), i32,
@@ -398,6 +401,27 @@ def viscache_decode_attention(batch: Batch, params: vc_params, layer: int, q: to
     _check("viscache_decode_attention", lib().viscache_decode_attention(
         ctypes.byref(batch.c), ctypes.byref(params), int(layer), _ptr(q), _ptr(K_out), _ptr(V_out),
         _ptr(K_text), _ptr(V_text), nt, _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
+    return out
+
+
+def viscache_decode_attention_kv4(batch: Batch, params: vc_params, layer: int, q: torch.Tensor,
+                                  kv4, K_text: Optional[torch.Tensor] = None,
+                                  V_text: Optional[torch.Tensor] = None, n_text: Optional[Sequence[int]] = None,
+                                  out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                                  stream=None) -> torch.Tensor:
+    """Decode step in `layer` over the 4-bit cache kv4 = (K_codes, V_codes, K_params, V_params)."""
+    if out is None:
+        out = torch.empty_like(q)
+    nt = _i32(n_text) if n_text is not None else None
+    if ws is None:
+        need = lib().viscache_decode_workspace_size(ctypes.byref(batch.c), ctypes.byref(params), nt)
+        if need == 0:
+            raise VisCacheError("viscache_decode_workspace_size", VC_ERR_INVALID_ARG)
+        ws = _workspace(need, q.device, None)
+    kc, vc_, kp, vp_ = kv4
+    _check("viscache_decode_attention_kv4", lib().viscache_decode_attention_kv4(
+        ctypes.byref(batch.c), ctypes.byref(params), int(layer), _ptr(q), _ptr(kc), _ptr(vc_), _ptr(kp),
+        _ptr(vp_), _ptr(K_text), _ptr(V_text), nt, _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
     return out
 
 

@@ -201,3 +201,68 @@ def test_many_splits_merge():
                                 Kt.double().numpy().reshape(Hkv, T, d), Vt.double().numpy().reshape(Hkv, T, d))
     err = np.abs(out[0].float().cpu().numpy() - ref)
     assert (err <= tolerance(torch.bfloat16, ref, float(V.abs().max()))).all()
+
+
+def _oracle_reconstruction(K, V, Bs, Hkv):
+    """The oracle's 4-bit reconstruction of a compacted cache, rounded to bf16."""
+    from oracle import quant as oq
+    K32, V32 = K.float().numpy(), V.float().numpy()
+    kc, vcodes, kp, vp = oq.quantize_cache(K32, V32, Bs, Hkv)
+    Kh = np.zeros_like(K32)
+    for row0, b in oq.segments(Bs, Hkv):
+        if b:
+            c, s, m = oq.quantize_keys(K32[row0:row0 + b])
+            Kh[row0:row0 + b] = oq.dequantize_keys(c, s, m)
+    Vh = oq.dequantize_values(oq.unpack(vcodes), vp[..., 0], vp[..., 1])
+    return torch.from_numpy(Kh).to(torch.bfloat16), torch.from_numpy(Vh).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_decode_over_4bit_cache_matches_oracle(d):
+    # the ragged batch of the bf16 test, its visual rows in 4-bit form
+    ns, rrs, texts, L, Hkv, Hq = [1500, 40, 333], [(25, 100), (50, 100), (19, 100)], [37, 0, 700], 4, 4, 28
+    batch = vc.Batch(ns, [8] * 3, rrs)
+    params = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    Bs = [budgets(L, n, rr) for n, rr in zip(ns, rrs)]
+    rows = sum(Hkv * sum(B) for B in Bs)
+    K = _rand((rows, d), 71, torch.bfloat16)
+    V = _rand((rows, d), 72, torch.bfloat16)
+    trows = sum(Hkv * t for t in texts)
+    Kt = _rand((trows, d), 73, torch.bfloat16)
+    Vt = _rand((trows, d), 74, torch.bfloat16)
+    kv4 = vc.viscache_kv4_quantize(batch, params, K.to(DEV), V.to(DEV))
+    Kh, Vh = _oracle_reconstruction(K, V, Bs, Hkv)
+    Kh64, Vh64 = Kh.double().numpy(), Vh.double().numpy()
+    Kt64, Vt64 = Kt.double().numpy(), Vt.double().numpy()
+    Ktd, Vtd = Kt.to(DEV), Vt.to(DEV)
+    gKh, gVh = vc.viscache_kv4_dequantize(batch, params, *kv4)
+    for l in range(L):
+        q = _rand((3, Hq, d), 80 + l, torch.bfloat16)
+        out = vc.viscache_decode_attention_kv4(batch, params, l, q.to(DEV), kv4, Ktd, Vtd, texts)
+        # same rows in bf16 through the bf16 kernel: identical arithmetic
+        ref_gpu = vc.viscache_decode_attention(batch, params, l, q.to(DEV), gKh, gVh, Ktd, Vtd, texts)
+        assert torch.equal(out, ref_gpu)
+        got = out.float().cpu().numpy()
+        r0, t0 = 0, 0
+        for r, B in enumerate(Bs):
+            v0 = r0 + Hkv * sum(B[:l])
+            Kv = Kh64[v0:v0 + Hkv * B[l]].reshape(Hkv, B[l], d)
+            Vv = Vh64[v0:v0 + Hkv * B[l]].reshape(Hkv, B[l], d)
+            T = texts[r]
+            Ktr = Kt64[t0:t0 + Hkv * T].reshape(Hkv, T, d)
+            Vtr = Vt64[t0:t0 + Hkv * T].reshape(Hkv, T, d)
+            ref = odec.decode_attention(q[r].double().numpy(), Kv, Vv, Ktr, Vtr)
+            vmax = max(np.abs(Vv).max(initial=0.0), np.abs(Vtr).max(initial=0.0), 1.0)
+            err = np.abs(got[r] - ref)
+            assert (err <= tolerance(torch.bfloat16, ref, vmax)).all(), "layer %d request %d" % (l, r)
+            r0 += Hkv * sum(B)
+            t0 += Hkv * T
+
+
+def test_decode_over_4bit_cache_rejects_fp32():
+    batch = vc.Batch([100], [8], [(25, 100)])
+    params = vc.make_params(2, 8, 2, 64, vc.VC_F32)
+    z = torch.zeros(4096, dtype=torch.uint8, device=DEV)
+    zf = torch.zeros(4096, dtype=torch.float32, device=DEV)
+    with pytest.raises(vc.VisCacheError):
+        vc.viscache_decode_attention_kv4(batch, params, 0, torch.zeros((1, 8, 64), device=DEV), (z, z, zf, zf))

@@ -508,12 +508,7 @@ def run_decode(args):
         # one cache alone (a profiling run): its time and kernel split only
         ms, kern, launches = res[names[0]]
         print(json.dumps({"stage": "decode", "cache": names[0], "requests": n_req, "ms_per_step": ms,
-                          "kv4_cache": {"ms_per_step": ms_q4, "value": n_req / (ms_q4 * 1e-3),
-                      "speedup_vs_compressed": ms / ms_q4, "kernels_ms_per_step": kern_q4,
-                      "cache_bytes_per_step": int(sum(n_req * Hkv * b for b in B) * (d + d // 32 * 8)
-                                                  + sum(n_req * Hkv * -(-b // 32) * d * 8 for b in B)
-                                                  + L * n_req * Hkv * T * d * 2 * 2)},
-        "kernels_ms_per_step": kern, "launches_per_step": launches, "clocks": clk}))
+                          "kernels_ms_per_step": kern, "launches_per_step": launches, "clocks": clk}))
         return
     ms, kern, launches = res["compressed"]
     ms_full, kern_full, _ = res["full"]

@@ -343,8 +343,9 @@ __device__ __forceinline__ UnitRows unit_rows(const DecodeTable& tb, int unit) {
   return x;
 }
 
-// Stage rows [0, nk) of a split (visual, then text) and zeros up to the next
-// 16-row boundary, so that the last MMA tile reads finite values.  Thread t
+// Stage rows [first, last) of a split's rows [0, nk) (visual, then text) and
+// zeros up to the next 16-row boundary, so that the last MMA tile reads
+// finite values.  Thread t
 // copies piece column t % PR of rows t / PR + k * (threads / PR); that row
 // step is a multiple of 8, so the column's XOR slot is the same for all of the
 // thread's rows.  `zsrc` is any valid device address: the zero-filling copies
@@ -352,12 +353,13 @@ __device__ __forceinline__ UnitRows unit_rows(const DecodeTable& tb, int unit) {
 template <int D>
 __device__ __forceinline__ void stage_split(uint32_t buf_s, const __nv_bfloat16* vis,
                                             const __nv_bfloat16* txt, int nv, int nk,
-                                            const __nv_bfloat16* zsrc, int first = 0) {
+                                            const __nv_bfloat16* zsrc, int first = 0,
+                                            int last = kSplitM) {
   using C = MmaCfg<D>;
   constexpr int RSTEP = kDecThreads / C::PR;
   static_assert(RSTEP % 8 == 0, "row step keeps the XOR slot");
   const int c = (int)threadIdx.x % C::PR, r0 = (int)threadIdx.x / C::PR;
-  const int rows = min(kSplitM, (nk + 15) & ~15);
+  const int rows = min(last, min(kSplitM, (nk + 15) & ~15));
   const uint32_t dst0 = buf_s + r0 * C::RB + mma_slot(r0, c) * 16;
   int r = r0;                                   // first row >= `first` in this thread's column
   if (first > r0) r += (first - r0 + RSTEP - 1) / RSTEP * RSTEP;
@@ -469,12 +471,27 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   const int unit = blockIdx.x;
   const UnitRows cur = unit_rows(tb, unit);
   const int nk = cur.nk;
-  if (Q4) stage_split<D>(buf_s, Kc, Kt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
-  else stage_split<D>(buf_s, Kc + cur.vis0 * D, Kt + cur.txt0 * D, cur.nv, nk, q);
-  stage_q<D>(qbuf_s, q + ((int64_t)cur.r * tb.Hq + cur.g * G) * D, G);
-  tc::cp_async_commit();
-  if (Q4) expand_q4<D, true>(buf, Kq + cur.vis0 * (D / 2), Kqp + cur.kg * D * 2, cur.nv);
-  tc::cp_async_wait<0>();
+  // bf16 rows move in halves of kHalf rows, so that loads overlap the MMAs:
+  // K rows [0, kHalf) with the query rows, then K rows [kHalf, 2 kHalf); QK of
+  // the first half (tile w) runs while the second arrives; V rows [0, kHalf)
+  // load into the freed half during QK of the second half (tile w + 8), V rows
+  // [kHalf, 2 kHalf) during the softmax; PV takes the halves in turn.
+  constexpr int kHalf = kSplitM / 2;
+  static_assert(C::TPW == 2 && kHalf == 16 * kDecWarps, "QK tile h of every warp lies in half h");
+  if (Q4) {
+    stage_split<D>(buf_s, Kc, Kt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
+    stage_q<D>(qbuf_s, q + ((int64_t)cur.r * tb.Hq + cur.g * G) * D, G);
+    tc::cp_async_commit();
+    expand_q4<D, true>(buf, Kq + cur.vis0 * (D / 2), Kqp + cur.kg * D * 2, cur.nv);
+    tc::cp_async_wait<0>();
+  } else {
+    stage_split<D>(buf_s, Kc + cur.vis0 * D, Kt + cur.txt0 * D, cur.nv, nk, q, 0, kHalf);
+    stage_q<D>(qbuf_s, q + ((int64_t)cur.r * tb.Hq + cur.g * G) * D, G);
+    tc::cp_async_commit();
+    stage_split<D>(buf_s, Kc + cur.vis0 * D, Kt + cur.txt0 * D, cur.nv, nk, q, kHalf);
+    tc::cp_async_commit();
+    tc::cp_async_wait<1>();                     // K rows [0, kHalf) and the query rows
+  }
   __syncthreads();
   // B fragments of Q^T (k = dimension, n = query) in log2 units, high + low,
   // built once for the CTA: item (ks, hf, lane) of KSTEPS x 2 x 32
@@ -503,6 +520,13 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   bool live[C::TPW];
 #pragma unroll
   for (int h = 0; h < C::TPW; ++h) {
+    if (!Q4 && h == 1) {
+      __syncthreads();                          // K rows [0, kHalf) read: V rows there
+      stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q, 0, kHalf);
+      tc::cp_async_commit();
+      tc::cp_async_wait<1>();                   // K rows [kHalf, 2 kHalf)
+      __syncthreads();
+    }
     const int mt = warp + h * kDecWarps;
     live[h] = 16 * mt < nk;
 #pragma unroll
@@ -524,7 +548,7 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     tc::cp_async_commit();
     expand_q4<D, false>(buf, Vq + cur.vis0 * (D / 2), Vqp + cur.vis0 * (D / 32) * 2, cur.nv);
   } else {
-    stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q);
+    stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q, kHalf);
     tc::cp_async_commit();
   }
   // softmax over the split: lane holds keys (16 mt + gid, + 8) x queries (2 tig, + 1)
@@ -578,7 +602,8 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     wsum[warp * kGm + 2 * tig] = l0;
     wsum[warp * kGm + 2 * tig + 1] = l1;
   }
-  tc::cp_async_wait<0>();                       // V rows
+  if (Q4) tc::cp_async_wait<0>();               // V rows
+  else tc::cp_async_wait<1>();                  // V rows [0, kHalf)
   __syncthreads();
   if (t < G) {
     float M = wmax[t], L = 0.f;
@@ -594,7 +619,7 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   float oacc[4] = {0.f, 0.f, 0.f, 0.f};
   const int steps = (nk + 15) >> 4;
   const int mi = lane >> 3;
-  for (int j = kw; j < steps; j += C::WPT) {
+  auto pv_step = [&](int j) {
     const int row = 16 * j + (lane & 7) + (mi >> 1) * 8;
     uint32_t a[4];
     ldsm_x4_t(buf_s + row * C::RB + mma_slot(row, 2 * dt + (mi & 1)) * 16, a);
@@ -605,7 +630,14 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     const uint32_t bl1 = *reinterpret_cast<const uint32_t*>(p_lo + gid * kPsLd + kb + 8);
     mma_bf16(oacc, a, bh0, bh1);
     mma_bf16(oacc, a, bl0, bl1);
+  };
+  constexpr int kHalfSteps = kHalf / 16;
+  for (int j = kw; j < min(steps, kHalfSteps); j += C::WPT) pv_step(j);
+  if (!Q4) {
+    tc::cp_async_wait<0>();                     // V rows [kHalf, 2 kHalf)
+    __syncthreads();
   }
+  for (int j = kHalfSteps + kw % C::WPT; j < steps; j += C::WPT) pv_step(j);
   // oacc: O[query 2 tig (+1)][dimension 16 dt + gid (+8)]
   float* po = part_o + (int64_t)unit * kGm * D;
   const int q0 = 2 * tig;

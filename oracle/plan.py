@@ -11,7 +11,7 @@ Allocation"; Sec. 4 "Implementation Details"; Algorithm 1 step 2):
 * RR = p * q * (h/L) * m with p = 1 here (no frame filtering), defaults
   h = 3L/4, m = 0.75                                                     (Sec. 4).
 
-Readings where the paper is silent (each listed in the design doc):
+Readings where the paper is silent:
 
 * total kept (token, layer) pairs per KV head  T = round(RR * n * L), so that
   sum_l B_l equals the stated retention times tokens times layers;

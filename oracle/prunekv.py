@@ -11,7 +11,7 @@ reads (widened).  Shapes, per request:
 
 GQA: query head j reads KV head j // G, G = Hq / Hkv.
 
-Readings where the paper is silent or ambiguous (listed in the design doc):
+Readings where the paper is silent or ambiguous:
 
 * the query rows of Eq. (token_score) are the W window rows;
 * the softmax of A^l runs over the n visual keys with scale 1/sqrt(d)

@@ -11,7 +11,7 @@ score of a candidate frame f given the selected set Omega is
 sim the cosine similarity; the highest-scoring frame joins Omega until the
 frame retention ratio p is reached (lambda = 0.7 in Sec. 4).
 
-Readings where the paper is silent (listed in the design doc):
+Readings where the paper is silent:
 
 * the redundancy term is 0 while Omega is empty, so the first frame is the
   most prompt-relevant one;

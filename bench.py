@@ -576,7 +576,8 @@ def run_decode(args):
                                                   + L * n_req * Hkv * T * d * 2 * 2)},
         "kernels_ms_per_step": kern,
         "roofline": {"kernel": main_kernel, "bound": "hbm", "achieved": achieved,
-                     "peak": pk["hbm"], "unit": "GB/s", "frac": achieved / pk["hbm"], "traffic": None,
+                     "peak": pk["hbm"], "unit": "GB/s", "frac": achieved / pk["hbm"],
+                     "traffic": traffic_for(main_kernel),
                      "peak_source": pk["source"]},
         "cpu_baseline": {"value": cpu, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
                          "sample": "%d single-request steps over all %d layers (fp64 numpy)" % (nr, L)},

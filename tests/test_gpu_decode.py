@@ -266,3 +266,46 @@ def test_decode_over_4bit_cache_rejects_fp32():
     zf = torch.zeros(4096, dtype=torch.float32, device=DEV)
     with pytest.raises(vc.VisCacheError):
         vc.viscache_decode_attention_kv4(batch, params, 0, torch.zeros((1, 8, 64), device=DEV), (z, z, zf, zf))
+
+
+def test_full_table_of_256_requests():
+    # the decode table's limit: 256 requests, mixed budgets, text lengths
+    # (some zero) and an evicted layer; also through the 4-bit path
+    n_req, L, Hkv, Hq, d = 256, 4, 2, 8, 64
+    ns = [24 + (37 * i) % 200 for i in range(n_req)]
+    rrs = [(25 + (i % 3) * 10, 100) for i in range(n_req)]
+    texts = [(11 * i) % 40 if i % 5 else 0 for i in range(n_req)]
+    batch = vc.Batch(ns, [8] * n_req, rrs)
+    params = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    Bs = [budgets(L, n, rr) for n, rr in zip(ns, rrs)]
+    rows = sum(Hkv * sum(B) for B in Bs)
+    K = _rand((rows, d), 91, torch.bfloat16)
+    V = _rand((rows, d), 92, torch.bfloat16)
+    trows = sum(Hkv * t for t in texts)
+    Kt = _rand((trows, d), 93, torch.bfloat16)
+    Vt = _rand((trows, d), 94, torch.bfloat16)
+    Kd, Vd, Ktd, Vtd = (x.to(DEV) for x in (K, V, Kt, Vt))
+    kv4 = vc.viscache_kv4_quantize(batch, params, Kd, Vd)
+    Kh, Vh = vc.viscache_kv4_dequantize(batch, params, *kv4)
+    K64, V64, Kt64, Vt64 = (x.double().numpy() for x in (K, V, Kt, Vt))
+    for l in (0, L - 1):
+        q = _rand((n_req, Hq, d), 95 + l, torch.bfloat16)
+        out = vc.viscache_decode_attention(batch, params, l, q.to(DEV), Kd, Vd, Ktd, Vtd, texts)
+        out4 = vc.viscache_decode_attention_kv4(batch, params, l, q.to(DEV), kv4, Ktd, Vtd, texts)
+        assert torch.equal(out4, vc.viscache_decode_attention(batch, params, l, q.to(DEV), Kh, Vh, Ktd, Vtd, texts))
+        got = out.float().cpu().numpy()
+        r0, t0 = 0, 0
+        for r, B in enumerate(Bs):
+            v0 = r0 + Hkv * sum(B[:l])
+            Kv = K64[v0:v0 + Hkv * B[l]].reshape(Hkv, B[l], d)
+            Vv = V64[v0:v0 + Hkv * B[l]].reshape(Hkv, B[l], d)
+            T = texts[r]
+            Ktr = Kt64[t0:t0 + Hkv * T].reshape(Hkv, T, d)
+            Vtr = Vt64[t0:t0 + Hkv * T].reshape(Hkv, T, d)
+            ref = odec.decode_attention(q[r].double().numpy(), Kv, Vv, Ktr, Vtr)
+            vmax = max(np.abs(Vv).max(initial=0.0), np.abs(Vtr).max(initial=0.0), 1.0)
+            assert (np.abs(got[r] - ref) <= tolerance(torch.bfloat16, ref, vmax)).all(), "layer %d request %d" % (l, r)
+            if B[l] + T == 0:
+                assert not got[r].any()
+            r0 += Hkv * sum(B)
+            t0 += Hkv * T

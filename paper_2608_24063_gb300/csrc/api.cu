@@ -673,10 +673,17 @@ size_t viscache_decode_workspace_size(const vc_batch* batch, const vc_params* p,
   std::vector<RequestPlan> plans;
   if (plan_batch(batch, p, &plans) != VC_OK) return 0;
   static thread_local DecodeTable tb;
+  if (decode_table(p, plans, 0, n_text, &tb) != VC_OK) return 0;   // checks the batch once
+  // the largest layer's (KV head, split) units, counted as decode_table does
+  const int64_t split = decode_split_keys(p->dtype);
   int64_t units = 0;
   for (int l = 0; l < p->L; ++l) {
-    if (decode_table(p, plans, l, n_text, &tb) != VC_OK) return 0;
-    units = std::max<int64_t>(units, tb.units);
+    int64_t u = 0;
+    for (size_t r = 0; r < plans.size(); ++r) {
+      const int64_t keys = plans[r].B[l] + (int64_t)(n_text ? n_text[r] : 0);
+      u += (int64_t)p->Hkv * std::max<int64_t>(1, (keys + split - 1) / split);
+    }
+    units = std::max(units, u);
   }
   return decode_ws(units, p->d, batch->n_req * p->Hkv).total;
 }

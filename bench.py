@@ -724,6 +724,10 @@ def run_quant(args):
 
 def main():
     args = parse()
+    if args.stage != "prunekv" and int(os.environ.get("RANK", "0")) != 0:
+        # the scout, decode and quantisation stages are single-GPU measurements:
+        # under torchrun the other ranks leave without work, rank 0 prints
+        return
     if args.stage == "quant":
         run_quant(args)
         return

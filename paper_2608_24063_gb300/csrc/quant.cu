@@ -10,12 +10,12 @@
 // channel in the low nibble; parameters are fp32 (scale, min) pairs.  The
 // code is decided in fp32 with IEEE subtraction and division and rint.
 //
-// One warp per key group (up to 32 rows of one segment), lane t owning d/32
-// adjacent channels (vector loads of a row's piece, the codes stored as one
-// 8- or 16-bit word): the key statistics per channel over the group's rows,
-// the value statistics per row from the lanes of each 32-channel group (xor
-// shuffles).  The work is a streaming pass (read 2 x 2 bytes, write
-// 2 x ~0.75 bytes per element pair): HBM-bound.
+// One warp per key group (up to 32 rows of one segment): for the keys lane t
+// owns d/32 adjacent channels (vector loads of a row's piece, the codes
+// stored as one 8- or 16-bit word, statistics per channel over the group's
+// rows); for the values a lane owns one (row, 32-channel group) pair at a
+// time (16-byte loads, its own statistics, 16 bytes of codes).  The work is a
+// streaming pass (read 2 x 2 bytes, write 2 x ~0.75 bytes per element pair).
 #include <cuda_bf16.h>
 #include <stdint.h>
 
@@ -125,15 +125,14 @@ __device__ __forceinline__ void store_codes(uint8_t* dst, const uint32_t (&q)[CP
 }
 
 // One warp per key group: lane t owns channels CPT t .. CPT t + CPT - 1 of the
-// group's rows.  Keys: a pass over the rows for the per-channel minimum and
-// maximum, then a second pass (the rows are cache-resident) for the codes.
-// Values: row by row, the TPG = 32 / CPT lanes of a 32-channel group combine
-// their minima and maxima with xor shuffles.
+// group's rows for the keys (a pass over the rows for the per-channel minimum
+// and maximum, then a second pass, the rows cache-resident, for the codes);
+// for the values each lane takes whole (row, 32-channel group) pairs.
 template <typename T, int D>
 __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
     const __grid_constant__ QuantTable tb, int units, const T* __restrict__ K, const T* __restrict__ V,
     uint8_t* __restrict__ Kc, uint8_t* __restrict__ Vc, float2* __restrict__ Kp, float2* __restrict__ Vp) {
-  constexpr int CPT = D / 32, TPG = kGroup / CPT;
+  constexpr int CPT = D / 32;
   const int unit = blockIdx.x * kQuantWarps + (threadIdx.x >> 5);
   if (unit >= units) return;
   const int lane = threadIdx.x & 31, c0 = lane * CPT;
@@ -172,31 +171,38 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
     for (int j = 0; j < CPT; ++j) q[j] = code_of(v[j], mn[j], ks[j], ki[j]);
     store_codes<CPT>(kc + i * (D / 2), q);
   }
-  const T* vp = V + gr.row * D + c0;
-  uint8_t* vc = Vc + gr.row * (D / 2) + c0 / 2;
-  float2* vpar = Vp + gr.row * (D / kGroup) + lane / TPG;
-#pragma unroll 4
-  for (int i = 0; i < gr.nrows; ++i) {
-    float v[CPT];
-    load_cpt<T, CPT>(vp + i * D, v);
+  // values: lane (row i, 32-channel group gv) takes the group whole (NG groups
+  // a row, 32 / NG rows a pass): 16-byte loads, its own minimum and maximum,
+  // 16 bytes of codes
+  constexpr int NG = D / kGroup, RPP = 32 / NG;
+  const int gv = lane % NG;
+  for (int i = lane / NG; i < gr.nrows; i += RPP) {
+    float v[kGroup];
+    const T* src = V + (gr.row + i) * D + gv * kGroup;
+#pragma unroll
+    for (int k = 0; k < kGroup; k += CPT) {
+      float u[CPT];
+      load_cpt<T, CPT>(src + k, u);
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) v[k + j] = u[j];
+    }
     float lo = v[0], hi = v[0];
 #pragma unroll
-    for (int j = 1; j < CPT; ++j) {
-      lo = fminf(lo, v[j]);
-      hi = fmaxf(hi, v[j]);
-    }
-#pragma unroll
-    for (int o = 1; o < TPG; o <<= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+    for (int k = 1; k < kGroup; ++k) {
+      lo = fminf(lo, v[k]);
+      hi = fmaxf(hi, v[k]);
     }
     const float vs = __fdiv_rn(__fsub_rn(hi, lo), 15.f);
     const float vi = vs > 0.f ? __frcp_rn(vs) : 0.f;
-    if (lane % TPG == 0) vpar[i * (D / kGroup)] = make_float2(vs, lo);
-    uint32_t q[CPT];
+    Vp[(gr.row + i) * NG + gv] = make_float2(vs, lo);
+    uint32_t w[4];
 #pragma unroll
-    for (int j = 0; j < CPT; ++j) q[j] = code_of(v[j], lo, vs, vi);
-    store_codes<CPT>(vc + i * (D / 2), q);
+    for (int b = 0; b < 4; ++b) {
+      w[b] = 0u;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) w[b] |= code_of(v[8 * b + k], lo, vs, vi) << (4 * k);
+    }
+    *reinterpret_cast<uint4*>(Vc + (gr.row + i) * (D / 2) + gv * (kGroup / 2)) = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 

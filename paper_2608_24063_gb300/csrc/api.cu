@@ -379,6 +379,22 @@ int plan_batch(const vc_batch* b, const vc_params* p, std::vector<RequestPlan>* 
     return VC_ERR_INVALID_ARG;
   if (p->schedule < VC_SCHED_PARABOLA || p->schedule > VC_SCHED_GEOMETRIC) return VC_ERR_INVALID_ARG;
   if (p->drop_mode != VC_DROP_SURVIVORS && p->drop_mode != VC_DROP_ALL) return VC_ERR_INVALID_ARG;
+  // The plans depend only on these numbers; a caller that repeats a batch (a
+  // decode step calls once per layer) gets the previous plans back.
+  thread_local std::vector<int64_t> last_key;
+  thread_local std::vector<RequestPlan> last_plans;
+  std::vector<int64_t> key = {b->n_req, p->L, p->h, p->m_num, p->m_den, p->schedule, p->drop_mode};
+  key.reserve(key.size() + 4 * (size_t)b->n_req);
+  for (int r = 0; r < b->n_req; ++r) {
+    key.push_back(b->n_vis[r]);
+    key.push_back(b->W[r]);
+    key.push_back(b->rr_num[r]);
+    key.push_back(b->rr_den[r]);
+  }
+  if (key == last_key) {
+    *plans = last_plans;
+    return VC_OK;
+  }
   plans->assign(b->n_req, RequestPlan{});
   for (int r = 0; r < b->n_req; ++r) {
     RequestPlan& q = (*plans)[r];
@@ -391,6 +407,8 @@ int plan_batch(const vc_batch* b, const vc_params* p, std::vector<RequestPlan>* 
                                             &q.h);
     if (rc != VC_OK) return rc;
   }
+  last_key.swap(key);
+  last_plans = *plans;
   return VC_OK;
 }
 

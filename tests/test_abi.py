@@ -193,3 +193,23 @@ def test_kv4_entries_reject_bad_arguments_without_touching_the_device():
     assert lib.viscache_kv4_dequantize(*args(p, p, p, p, None, p, None)) == vc.VC_ERR_INVALID_ARG
     bad = vc.make_params(4, 8, 2, 96, vc.VC_BF16)
     assert lib.viscache_kv4_sizes(ctypes.byref(b.c), ctypes.byref(bad), None, None) == vc.VC_ERR_INVALID_ARG
+
+
+def test_repeated_batches_reuse_plans_and_changes_replan():
+    # the batch entry points plan once per distinct (batch, parameters); any
+    # change of either must give the new plan, alternating calls included
+    b1 = vc.Batch([12544, 700], [64, 8], [(19, 100), (25, 100)])
+    b2 = vc.Batch([12544, 701], [64, 8], [(19, 100), (25, 100)])
+    p1 = vc.make_params(28, 28, 4, 128, vc.VC_BF16)
+    p2 = vc.make_params(28, 28, 4, 128, vc.VC_BF16, schedule=vc.VC_SCHED_FIXED)
+
+    def expect(b, p):
+        rows = groups = 0
+        for n, (a, d) in zip(b.n_vis, b.rr):
+            B = plan.plan_budgets(28, n, Fraction(a, d), schedule="fixed" if p.schedule else "parabola")[0]
+            rows += 4 * sum(B)
+            groups += 4 * sum(-(-x // 32) for x in B)
+        return rows, groups
+
+    for b, p in [(b1, p1), (b1, p1), (b2, p1), (b1, p1), (b1, p2), (b1, p1), (b2, p2)]:
+        assert vc.viscache_kv4_sizes(b, p) == expect(b, p)

@@ -66,3 +66,20 @@ def test_gqa_map_contiguous_groups(G):
         alone = decode.decode_attention(q[j:j + 1], K[g:g + 1], V[g:g + 1])[0]
         np.testing.assert_allclose(base[j], alone, rtol=1e-13, atol=1e-14)
     assert not np.allclose(base, got) or Hkv == 1
+
+
+def test_two_keys_closed_form():
+    # keys k1, k2 with scaled logits differing by delta: the output is the
+    # logistic mix sigma(delta) v1 + (1 - sigma(delta)) v2, whatever d is
+    d = 16
+    q = np.zeros((1, d))
+    q[0, 0] = 2.0
+    K = np.zeros((1, 2, d))
+    K[0, 0, 0] = 3.0                      # logit 6 / sqrt(16) = 1.5
+    K[0, 1, 0] = -1.0                     # logit -2 / 4 = -0.5
+    V = np.zeros((1, 2, d))
+    V[0, 0, :] = 1.0
+    V[0, 1, :] = -3.0
+    w = 1.0 / (1.0 + np.exp(-2.0))        # delta = 2
+    got = decode.decode_attention(q, K, V)
+    np.testing.assert_allclose(got[0], w * 1.0 + (1 - w) * -3.0, rtol=0, atol=1e-15)

@@ -36,7 +36,10 @@
  *   ascending original position.  Layers l > h (B_l = 0) are absent.
  *   Drop lists use the same scheme with D_l = Nq - B_l (l <= h, B_l > 0).
  * - Supported: d in {64, 128}; 1 <= n <= 65536; W >= 1; Hq % Hkv == 0;
- *   L <= 256.  The library is stateless and thread-safe.
+ *   L <= 256.  The library is thread-safe.  Its only state is per host
+ *   thread (the last batch's budget plans, reused when the next call repeats
+ *   the batch and parameters; results never depend on it) plus the kernel-path
+ *   switch and the profiling switch below.
  */
 #ifndef VISCACHE_H_
 #define VISCACHE_H_

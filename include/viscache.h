@@ -38,8 +38,11 @@
  * - Supported: d in {64, 128}; 1 <= n <= 65536; W >= 1; Hq % Hkv == 0;
  *   L <= 256.  The library is thread-safe.  Its only state is per host
  *   thread (the last batch's budget plans, reused when the next call repeats
- *   the batch and parameters; results never depend on it) plus the kernel-path
- *   switch and the profiling switch below.
+ *   the batch and parameters; results never depend on it), the kernel-path
+ *   switch and the profiling switch below, and the fixed scratch array of
+ *   prunekv_score_static (VC_STATIC_SCRATCH_BYTES on every device that loads
+ *   the library) with its process-wide cache of that array's device address
+ *   per CUDA context.
  */
 #ifndef VISCACHE_H_
 #define VISCACHE_H_
@@ -154,31 +157,52 @@ int prunekv_score(const void* Qw, const void* K, int dtype, int32_t L, int32_t H
 
 /*
  * prunekv_score_static -- prunekv_score for callers that cannot allocate
- * device memory (code running inside an allocator or memory-pool hook, a
- * runtime that replays frozen CUDA graphs and hands out no workspace, an
- * embedding host without a device allocator).  The paper has no counterpart:
- * this is a deployment convenience, not a step of the method.
+ * device memory (code running inside an allocator or memory-pool hook, where
+ * a cudaMalloc would re-enter the allocator; a runtime that replays frozen
+ * CUDA graphs and hands out no workspace; an embedding host without a device
+ * allocator).  The paper has no counterpart: this is a deployment
+ * convenience, not a step of the method.
  *
  * Same arguments, arithmetic and result as prunekv_score, minus the
  * workspace: the scratch (status word, plan tables, per-row log-sum-exp) is a
  * fixed device array of VC_STATIC_SCRATCH_BYTES inside the library, which
- * every GPU that loads the library holds until the process exits.
+ * every GPU that loads the library holds until the process exits.  Nothing
+ * is allocated: no cudaMalloc, cudaFree or allocating library routine.
  *   - Problems needing more scratch than that (prunekv_score_workspace_size
- *     (L, Hq, W) > VC_STATIC_SCRATCH_BYTES, i.e. roughly L*Hq*W > 800,000
- *     window rows) are rejected with VC_ERR_WORKSPACE before any device work.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current and caches it; make
- *     that first call before capturing a stream.  Nothing is allocated.
+ *     (L, Hq, W) > VC_STATIC_SCRATCH_BYTES, i.e. roughly L*Hq*W > 460,000
+ *     window rows: the 7B shape with up to 512 window rows fits, the 72B
+ *     shape with 128 window rows, 655,360 rows, does not) are rejected with
+ *     VC_ERR_WORKSPACE before any device work.
+ *   - The first call in a CUDA context looks up the array's device address
+ *     (cudaGetSymbolAddress) with that context's device current and caches
+ *     it with the context's id; make that first call before capturing a
+ *     stream.  After cudaDeviceReset (or when the primary context is
+ *     released and created again) the array may move: the next call sees a
+ *     new context id and looks the address up again, so it too should come
+ *     before any capture.
  *   - All calls on a device share the array and it keeps the last call's
- *     contents; each call rewrites everything it reads.  Calls whose kernels
- *     overlap on the GPU race on the array: serialise them.
- *   - Device-side status is kept in the shared array and is not reported;
- *     the return value covers arguments and launches.
+ *     contents; each call rewrites everything it reads (the status word is
+ *     cleared when the call starts).  Calls whose kernels overlap on the GPU
+ *     race on the array: serialise them.
+ *   - Device-side errors (a bounded wait that gave up, an index out of
+ *     range) land in the array's status word: prunekv_score_static_status
+ *     reads it after the call, exactly as prunekv_get_status does for a
+ *     workspace.
  */
 #define VC_STATIC_SCRATCH_BYTES (16u << 20)
 int prunekv_score_static(const void* Qw, const void* K, int dtype, int32_t L, int32_t Hq,
                          int32_t Hkv, int32_t d, int32_t n_vis, int32_t W, float scale,
                          int rank_mode, const float* row_lse, float* scores, void* stream);
+/* Size in bytes of prunekv_score_static's scratch array (VC_STATIC_SCRATCH_BYTES). */
+size_t prunekv_score_static_capacity(void);
+/*
+ * Device-side status of the last prunekv_score_static call on the current
+ * device: synchronises `stream` (pass the stream the call used), then returns
+ * VC_OK, the first device error the call recorded (VC_ERR_DEVICE_TIMEOUT,
+ * VC_ERR_DEVICE_INDEX), or VC_ERR_CUDA if the word could not be read.
+ * Allocates nothing.
+ */
+int prunekv_score_static_status(void* stream);
 
 /*
  * prunekv_select -- rank, keep and drop sets, Algorithm 1 steps 1 and 3.
@@ -291,6 +315,13 @@ int prunekv_compress(const vc_batch* batch, const vc_params* p, const void* Qw,
  * VC_ERR_WORKSPACE, VC_ERR_CUDA.
  */
 size_t viscache_scout_workspace_size(int32_t n_req, const int32_t* n_frames, int32_t D);
+/*
+ * viscache_scout_sizes -- host only: the number of keyframes k_r = ceil(p * F_r)
+ * viscache_scout_mmr picks for each video (the rows its outputs need), written
+ * to k_out (host int32 [n_req]).  Same argument checks as viscache_scout_mmr.
+ */
+int viscache_scout_sizes(int32_t n_req, const int32_t* n_frames, uint32_t p_num, uint32_t p_den,
+                         int32_t* k_out);
 int viscache_scout_mmr(const float* H, const float* prompt, int32_t n_req, const int32_t* n_frames,
                        int32_t D, float lambda, uint32_t p_num, uint32_t p_den, int32_t* order_out,
                        int32_t* keyframes_out, float* gains_out, int32_t* k_out, void* ws,

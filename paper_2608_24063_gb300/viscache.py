@@ -38,8 +38,9 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_select_workspace_size", "prunekv_select", "prunekv_fuse_workspace_size",
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
-            "viscache_profile_read", "prunekv_score_static", "viscache_set_kernel_path",
-            "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_mmr",
+            "viscache_profile_read", "prunekv_score_static", "prunekv_score_static_capacity",
+            "prunekv_score_static_status", "viscache_set_kernel_path",
+            "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_sizes", "viscache_scout_mmr",
             "viscache_decode_workspace_size", "viscache_decode_attention",
             "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize",
             "viscache_decode_attention_kv4")
@@ -82,6 +83,7 @@ def lib() -> ctypes.CDLL:
                                                pi32]
         L.viscache_scout_workspace_size.argtypes = [i32, pi32, i32]
         L.viscache_scout_workspace_size.restype = sz
+        L.viscache_scout_sizes.argtypes = [i32, pi32, u32, u32, pi32]
         L.viscache_scout_mmr.argtypes = [vp, vp, i32, pi32, i32, f32, u32, u32, vp, vp, vp, pi32, vp, sz, vp]
         L.viscache_kv4_sizes.argtypes = [ctypes.POINTER(vc_batch), ctypes.POINTER(vc_params),
                                          ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
@@ -101,6 +103,9 @@ def lib() -> ctypes.CDLL:
                                     vp, sz, vp]
         L.prunekv_score_static.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp,
                                            vp, vp]
+        L.prunekv_score_static_capacity.argtypes = []
+        L.prunekv_score_static_capacity.restype = sz
+        L.prunekv_score_static_status.argtypes = [vp]
         L.prunekv_select_workspace_size.argtypes = [i32, i32, i32, i32]
         L.prunekv_select_workspace_size.restype = sz
         L.prunekv_select.argtypes = [vp, i32, i32, i32, pi32, i32, i32, vp, vp, vp, vp, sz, vp]
@@ -210,7 +215,9 @@ def viscache_scout_mmr(H: torch.Tensor, prompt: torch.Tensor, n_frames: Sequence
     need = lib().viscache_scout_workspace_size(n_req, nf, D)
     if need == 0:
         raise VisCacheError("viscache_scout_workspace_size", VC_ERR_INVALID_ARG)
-    ks = [max(1, min(f, (p[0] * f + p[1] - 1) // p[1])) for f in n_frames]
+    kk = (ctypes.c_int32 * n_req)()
+    _check("viscache_scout_sizes", lib().viscache_scout_sizes(n_req, nf, p[0], p[1], kk))
+    ks = list(kk)
     dev = H.device
     if out is not None:
         order, keys, gains = out
@@ -251,7 +258,14 @@ def prunekv_score(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,
     return scores
 
 
-STATIC_SCRATCH_BYTES = 16 << 20
+def prunekv_score_static_capacity() -> int:
+    """Bytes of the library's fixed scratch array (VC_STATIC_SCRATCH_BYTES)."""
+    return lib().prunekv_score_static_capacity()
+
+
+def prunekv_score_static_status(stream=None) -> int:
+    """Device status of the last prunekv_score_static call (synchronises `stream`)."""
+    return lib().prunekv_score_static_status(_stream(stream))
 
 
 def prunekv_score_static(Qw: torch.Tensor, K: torch.Tensor, scale: float = 0.0,

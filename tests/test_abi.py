@@ -213,3 +213,33 @@ def test_repeated_batches_reuse_plans_and_changes_replan():
 
     for b, p in [(b1, p1), (b1, p1), (b2, p1), (b1, p1), (b1, p2), (b1, p1), (b2, p2)]:
         assert vc.viscache_kv4_sizes(b, p) == expect(b, p)
+
+
+def test_static_scratch_capacity_matches_header():
+    """The no-allocation scoring entry point's array size, as the library reports it,
+    is the header's VC_STATIC_SCRATCH_BYTES (the binding reads it from the library)."""
+    src = open(os.path.join(ROOT, "include", "viscache.h")).read()
+    m = re.search(r"#define\s+VC_STATIC_SCRATCH_BYTES\s+\((\d+)u\s*<<\s*(\d+)\)", src)
+    assert m, "VC_STATIC_SCRATCH_BYTES not found"
+    assert vc.prunekv_score_static_capacity() == int(m.group(1)) << int(m.group(2))
+    # the 7B shape fits with up to 512 window rows; the 72B shape with 128 does not
+    assert vc.prunekv_score_workspace_size(28, 28, 512) <= vc.prunekv_score_static_capacity()
+    assert vc.prunekv_score_workspace_size(80, 64, 128) > vc.prunekv_score_static_capacity()
+
+
+def test_scout_sizes_match_oracle_keyframe_count():
+    """The C sizing call the binding uses for the scout's outputs gives the oracle's
+    k = ceil(p F) for every video; bad arguments come back as codes."""
+    from oracle import scout as osc
+    frames = [1, 2, 3, 7, 64, 100, 333, 4096]
+    for p in [(1, 1), (3, 4), (1, 3), (2, 7), (1, 4096)]:
+        kk = (ctypes.c_int32 * len(frames))()
+        arr = (ctypes.c_int32 * len(frames))(*frames)
+        assert vc.lib().viscache_scout_sizes(len(frames), arr, p[0], p[1], kk) == vc.VC_OK
+        assert list(kk) == [osc.keyframe_count(F, Fraction(*p)) for F in frames], p
+    one = (ctypes.c_int32 * 1)(5)
+    out = (ctypes.c_int32 * 1)()
+    assert vc.lib().viscache_scout_sizes(1, one, 0, 4, out) == vc.VC_ERR_INVALID_ARG
+    assert vc.lib().viscache_scout_sizes(1, one, 5, 4, out) == vc.VC_ERR_INVALID_ARG
+    assert vc.lib().viscache_scout_sizes(1, (ctypes.c_int32 * 1)(0), 3, 4, out) == vc.VC_ERR_INVALID_ARG
+    assert vc.lib().viscache_scout_sizes(1, one, 3, 4, None) == vc.VC_ERR_INVALID_ARG

@@ -485,6 +485,17 @@ extern "C" size_t viscache_scout_workspace_size(int32_t n_req, const int32_t* n_
   return scout_plan(n_req, n_frames, D, 1, 1, 0.5f, &tb, &lay) == VC_OK ? lay.total : 0;
 }
 
+extern "C" int viscache_scout_sizes(int32_t n_req, const int32_t* n_frames, uint32_t p_num,
+                                    uint32_t p_den, int32_t* k_out) {
+  if (!k_out) return VC_ERR_INVALID_ARG;
+  ScoutTable tb;
+  ScoutLayout lay;
+  const int rc = scout_plan(n_req, n_frames, 1, p_num, p_den, 0.5f, &tb, &lay);
+  if (rc != VC_OK) return rc;
+  for (int r = 0; r < n_req; ++r) k_out[r] = tb.k[r];
+  return VC_OK;
+}
+
 extern "C" int viscache_scout_mmr(const float* H, const float* prompt, int32_t n_req,
                                   const int32_t* n_frames, int32_t D, float lambda, uint32_t p_num,
                                   uint32_t p_den, int32_t* order_out, int32_t* keyframes_out,

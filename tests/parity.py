@@ -23,6 +23,17 @@ def np64(t: torch.Tensor) -> np.ndarray:
     return t.detach().to("cpu", torch.float64).numpy()
 
 
+def check_v_rows(got, ref, tol, tag):
+    """V_out rows of one (layer, KV head) against the oracle's fusion (both float64):
+    max|d| <= tol max|ref| and |d| <= tol |ref| + tol rms(ref) elementwise."""
+    diff = np.abs(got - ref)
+    amax = float(np.abs(ref).max()) if ref.size else 0.0
+    rms = float(np.sqrt((ref ** 2).mean())) if ref.size else 0.0
+    assert float(diff.max(initial=0)) <= tol * amax + 1e-30, "V_out max %s: %g" % (tag, diff.max(initial=0))
+    bad = diff > tol * np.abs(ref) + tol * rms
+    assert not bad.any(), "V_out elementwise %s: %d bad" % (tag, int(bad.sum()))
+
+
 def check_sets(gpu_keep, ref_rank, s_ref, cut, log, tag):
     """gpu_keep: the GPU's top-`cut` set (ascending ints); ref_rank: oracle rank per token."""
     ref_keep = np.sort(np.argsort(ref_rank, kind="stable")[:cut])
@@ -86,13 +97,7 @@ def check_request(Qw, K, V, B, Nq, gpu, mu, tau, rank_mode="shared", scale=None,
             assert torch.equal(Kg[r0:r0 + b], K[l, g].cpu()[torch.from_numpy(kg)]), "K_out l=%d g=%d" % (l, g)
             if check_v:
                 ref = ok.fuse_values(Vn[l, g], kg, dg, mu, tau)
-                got = Vg[r0:r0 + b]
-                diff = np.abs(got - ref)
-                amax = float(np.abs(ref).max()) if ref.size else 0.0
-                rms = float(np.sqrt((ref ** 2).mean())) if ref.size else 0.0
-                assert float(diff.max(initial=0)) <= tol * amax + 1e-30, "V_out max l=%d g=%d: %g" % (l, g, diff.max())
-                bad = diff > tol * np.abs(ref) + tol * rms
-                assert not bad.any(), "V_out elementwise l=%d g=%d: %d bad" % (l, g, int(bad.sum()))
+                check_v_rows(Vg[r0:r0 + b], ref, tol, "l=%d g=%d" % (l, g))
         P += b
         Qd += D
     return log

@@ -245,11 +245,17 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
-def rank_workload(wl, rank):
-    """The workload one rank compresses under weak scaling: the same shapes and
-    request mix, its own requests (the seed offset by the rank)."""
-    import dataclasses
-    return wl if rank == 0 else dataclasses.replace(wl, seed=wl.seed + 7919 * rank)
+def rank_requests(wl, world, rank):
+    """Weak scaling: the job is `world` copies of the workload's requests (each copy
+    its own seeded values), split over the ranks by the work-balanced request
+    partition; no data-path collective.  Returns (job workload, this rank's request
+    indices, this rank's workload view).  At world = 1 the job is the workload."""
+    from paper_2608_24063_gb300 import shard, synth
+    job = synth.replicated(wl, world)
+    costs = [shard.request_cost(r.n, r.W, wl.L, wl.Hq) for r in job.requests]
+    mine = shard.partition_requests(costs, world)[rank]
+    view = synth.scaled(job, job.name, requests=[job.requests[i] for i in mine])
+    return job, mine, view
 
 
 def max_over_ranks(x, world, dist, device):
@@ -262,9 +268,9 @@ def max_over_ranks(x, world, dist, device):
     return float(t.item())
 
 
-def job_value(units_per_rank, world, ms_per_step):
-    """Whole-job throughput: units of all ranks / the slowest rank's step time."""
-    return world * units_per_rank / (ms_per_step * 1e-3)
+def job_value(units_all_ranks, ms_per_step):
+    """Whole-job throughput: the units of all ranks / the slowest rank's step time."""
+    return units_all_ranks / (ms_per_step * 1e-3)
 
 
 def workload_config(wl, args=None):
@@ -758,13 +764,15 @@ def main():
     st = torch.cuda.current_stream()
 
     # inputs: generated on the device, resident in HBM before timing
-    qs, ks, vs = synth.generate(rank_workload(wl, rank), dev)
+    job, mine, wl_rank = rank_requests(wl, world, rank)
+    job_units = sum(r.n * wl.L for r in job.requests)
+    qs, ks, vs = synth.generate(job, dev, mine)
     Q = torch.cat([q.flatten() for q in qs]) if len(qs) > 1 else qs[0]
     K = torch.cat([k.flatten() for k in ks]) if len(ks) > 1 else ks[0]
     V = torch.cat([v.flatten() for v in vs]) if len(vs) > 1 else vs[0]
     del qs, ks, vs
-    batch = vc.Batch([r.n for r in wl.requests], [r.W for r in wl.requests],
-                     [(r.rr_num, r.rr_den) for r in wl.requests])
+    batch = vc.Batch([r.n for r in wl_rank.requests], [r.W for r in wl_rank.requests],
+                     [(r.rr_num, r.rr_den) for r in wl_rank.requests])
     prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16 if wl.dtype == "bf16" else vc.VC_F32,
                          schedule=SCHEDULES[args.schedule], drop_mode=DROPS[args.drop],
                          rank_mode=vc.VC_RANK_PER_LAYER if args.rank == "per_layer" else vc.VC_RANK_SHARED)
@@ -836,9 +844,9 @@ def main():
     vc.viscache_profile_enable(False)
     assert vc.prunekv_get_status(ws) == vc.VC_OK
 
-    plans = plans_for(wl, vc, args.schedule, args.drop)
-    work = algorithmic(wl, plans)
-    value = job_value(work["tokens_layers"], world, ms_step)
+    plans = plans_for(wl_rank, vc, args.schedule, args.drop)
+    work = algorithmic(wl_rank, plans)
+    value = job_value(job_units, ms_step)
     pk = peaks()
 
     # dominant kernel
@@ -935,7 +943,7 @@ def main():
         assert torch.equal(oI[(e_steps - 1) % 2], dI[(e_steps - 1) % 2].cpu())
         ems = max_over_ranks(a.elapsed_time(b) / e_steps, world, dist, dev)
         v_bytes = work["surv_v_bytes"] if v_host else V.numel() * V.element_size()
-        e2e = {"value": job_value(work["tokens_layers"], world, ems), "unit": UNIT,
+        e2e = {"value": job_value(job_units, ems), "unit": UNIT,
                "ms_per_step": ems, "pipelined": "copy-in / compress / copy-out on three streams",
                "v_source": "pinned host memory read by the gather kernel (survivor rows only)"
                            if v_host else "copied to the device every step",

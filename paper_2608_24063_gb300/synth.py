@@ -313,10 +313,19 @@ def scaled(wl: Workload, name: str, *, L=None, Hq=None, Hkv=None, d=None, dtype=
         seed=wl.seed if seed is None else seed)
 
 
-def generate(wl: Workload, device="cpu"):
-    """All requests' (Qw, K, V) as lists of per-request tensors on ``device``."""
+def replicated(wl: Workload, copies: int) -> Workload:
+    """The workload's request list repeated `copies` times.  Request r draws from
+    its own streams (the request index is part of every stream key), so the copies
+    have the same shapes and structure and different values; copy 0 is `wl`'s own
+    requests, bit for bit."""
+    return dataclasses.replace(wl, requests=tuple(wl.requests) * copies)
+
+
+def generate(wl: Workload, device="cpu", indices: Optional[Sequence[int]] = None):
+    """Requests' (Qw, K, V) as lists of per-request tensors on ``device``: all of
+    them, or those with the given indices (in that order)."""
     qs, ks, vs = [], [], []
-    for r in range(len(wl.requests)):
+    for r in (range(len(wl.requests)) if indices is None else indices):
         q = make_q(wl, r, "cpu")
         k, v = make_kv(wl, r, q, device)
         qs.append(q.to(device))

@@ -826,10 +826,43 @@ def main():
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    clk = clocks.stop()
     ms = max_over_ranks(t0.elapsed_time(t1), world, dist, dev)
     ms_step = ms / args.steps
+    # the same K-step window repeated until ~1.5 s of load have run, with the
+    # clock sampler still going, so the clock record covers a long load; the
+    # headline stays the first window of exactly K steps
+    windows = []
+    if args.steps > 0:
+        n_more = max(0, min(2000, int(math.ceil(1500.0 / max(ms, 1e-3))) - 1))
+        ea = [torch.cuda.Event(enable_timing=True) for _ in range(n_more + 1)]
+        for i in range(n_more):
+            ea[i].record(st)
+            for _ in range(args.steps):
+                run()
+        ea[n_more].record(st)
+        torch.cuda.synchronize()
+        windows = [ea[i].elapsed_time(ea[i + 1]) / args.steps for i in range(n_more)]
+    clk = clocks.stop()
+    if clk is not None:
+        clk["window_s"] = round((ms + sum(windows) * args.steps) / 1e3, 3)
+    sustained = None
+    if windows:
+        sustained = {"windows": len(windows), "steps_per_window": args.steps,
+                     "ms_per_step_median": statistics.median(windows),
+                     "ms_per_step_min": min(windows), "ms_per_step_max": max(windows)}
     assert vc.prunekv_get_status(ws) == vc.VC_OK
+
+    # the same steps as direct calls (no graph, no per-kernel events)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(st)
+    for _ in range(args.steps):
+        step()
+    d1.record(st)
+    torch.cuda.synchronize()
+    ms_direct = max_over_ranks(d0.elapsed_time(d1), world, dist, dev) / max(args.steps, 1)
 
     # timed region 2: the same steps as direct calls with the library's event
     # pair around every kernel launch (per-kernel durations and launch count)
@@ -897,61 +930,67 @@ def main():
         dI = [idx, torch.empty_like(idx)]
         # V can stay in pinned host memory when the device reads it directly:
         # only the survivors' rows then cross to the GPU (read by the gather)
-        v_host = all(vc.viscache_device_accessible(t) for t in hV)
+        v_accessible = all(vc.viscache_device_accessible(t) for t in hV)
         s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
         ev = lambda: torch.cuda.Event()
         in_done, cmp_done, out_done = [ev(), ev()], [ev(), ev()], [ev(), ev()]
 
-        def e2e_step(i):
-            bsel = i % 2
-            if i >= 2:
-                s_in.wait_event(cmp_done[bsel])        # step i-2 has finished reading these inputs
-            with torch.cuda.stream(s_in):
-                dQ[bsel].copy_(hQ[bsel], non_blocking=True)
-                dK[bsel].copy_(hK[bsel], non_blocking=True)
-                if not v_host:
-                    dV[bsel].copy_(hV[bsel], non_blocking=True)
-                in_done[bsel].record(s_in)
-            s_cmp.wait_event(in_done[bsel])
-            if i >= 2:
-                s_cmp.wait_event(out_done[bsel])       # step i-2's outputs are back on the host
-            vc.prunekv_compress(batch, prm, dQ[bsel], dK[bsel], hV[bsel] if v_host else dV[bsel], dKo[bsel],
-                                dVo[bsel], dI[bsel], ws, stream=s_cmp)
-            cmp_done[bsel].record(s_cmp)
-            s_out.wait_event(cmp_done[bsel])
-            with torch.cuda.stream(s_out):
-                oK[bsel].copy_(dKo[bsel], non_blocking=True)
-                oV[bsel].copy_(dVo[bsel], non_blocking=True)
-                oI[bsel].copy_(dI[bsel], non_blocking=True)
-                out_done[bsel].record(s_out)
+        def measure_e2e(v_host):
+            def e2e_step(i):
+                bsel = i % 2
+                if i >= 2:
+                    s_in.wait_event(cmp_done[bsel])        # step i-2 has finished reading these inputs
+                with torch.cuda.stream(s_in):
+                    dQ[bsel].copy_(hQ[bsel], non_blocking=True)
+                    dK[bsel].copy_(hK[bsel], non_blocking=True)
+                    if not v_host:
+                        dV[bsel].copy_(hV[bsel], non_blocking=True)
+                    in_done[bsel].record(s_in)
+                s_cmp.wait_event(in_done[bsel])
+                if i >= 2:
+                    s_cmp.wait_event(out_done[bsel])       # step i-2's outputs are back on the host
+                vc.prunekv_compress(batch, prm, dQ[bsel], dK[bsel], hV[bsel] if v_host else dV[bsel],
+                                    dKo[bsel], dVo[bsel], dI[bsel], ws, stream=s_cmp)
+                cmp_done[bsel].record(s_cmp)
+                s_out.wait_event(cmp_done[bsel])
+                with torch.cuda.stream(s_out):
+                    oK[bsel].copy_(dKo[bsel], non_blocking=True)
+                    oV[bsel].copy_(dVo[bsel], non_blocking=True)
+                    oI[bsel].copy_(dI[bsel], non_blocking=True)
+                    out_done[bsel].record(s_out)
 
-        for i in range(4):
-            e2e_step(i)
-        torch.cuda.synchronize()
-        e_steps = max(4, min(args.steps, 12))
-        if world > 1:
-            dist.barrier()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(s_in)
-        for i in range(e_steps):
-            e2e_step(i)
-        s_out.wait_stream(s_in)
-        s_out.wait_stream(s_cmp)
-        b.record(s_out)
-        torch.cuda.synchronize()
-        assert vc.prunekv_get_status(ws) == vc.VC_OK
-        assert torch.equal(oI[(e_steps - 1) % 2], dI[(e_steps - 1) % 2].cpu())
-        ems = max_over_ranks(a.elapsed_time(b) / e_steps, world, dist, dev)
-        v_bytes = work["surv_v_bytes"] if v_host else V.numel() * V.element_size()
-        e2e = {"value": job_value(job_units, ems), "unit": UNIT,
-               "ms_per_step": ems, "pipelined": "copy-in / compress / copy-out on three streams",
-               "v_source": "pinned host memory read by the gather kernel (survivor rows only)"
-                           if v_host else "copied to the device every step",
-               "h2d_bytes_per_step": int(Q.numel() * Q.element_size() + K.numel() * K.element_size()
-                                         + v_bytes),
-               "d2h_bytes_per_step": int(K_out.numel() * K_out.element_size()
-                                         + V_out.numel() * V_out.element_size()
-                                         + idx.numel() * idx.element_size())}
+            for i in range(4):
+                e2e_step(i)
+            torch.cuda.synchronize()
+            e_steps = max(4, min(args.steps, 12))
+            if world > 1:
+                dist.barrier()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s_in)
+            for i in range(e_steps):
+                e2e_step(i)
+            s_out.wait_stream(s_in)
+            s_out.wait_stream(s_cmp)
+            b.record(s_out)
+            torch.cuda.synchronize()
+            assert vc.prunekv_get_status(ws) == vc.VC_OK
+            assert torch.equal(oI[(e_steps - 1) % 2], dI[(e_steps - 1) % 2].cpu())
+            ems = max_over_ranks(a.elapsed_time(b) / e_steps, world, dist, dev)
+            v_bytes = work["surv_v_bytes"] if v_host else V.numel() * V.element_size()
+            return {"value": job_value(job_units, ems), "unit": UNIT,
+                    "ms_per_step": ems, "pipelined": "copy-in / compress / copy-out on three streams",
+                    "v_source": "pinned host memory read by the gather kernel (survivor rows only)"
+                                if v_host else "copied to the device every step",
+                    "h2d_bytes_per_step": int(Q.numel() * Q.element_size() + K.numel() * K.element_size()
+                                              + v_bytes),
+                    "d2h_bytes_per_step": int(K_out.numel() * K_out.element_size()
+                                              + V_out.numel() * V_out.element_size()
+                                              + idx.numel() * idx.element_size())}
+
+        e2e = measure_e2e(v_accessible)
+        if v_accessible:
+            # beside it, every input copied to the device every step
+            e2e["full_copy"] = measure_e2e(False)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -972,6 +1011,7 @@ def main():
                 "data": "synthetic (seeded, structure of the paper's long-video workloads)",
                 "config": dict(workload_config(wl, args), launch="cuda graph of the prunekv_compress call"
                                if graph is not None else "direct prunekv_compress calls"),
+                "ms_per_step_direct": ms_direct, "sustained": sustained,
                 "roofline": roof, "pass_roofline": pass_roof,
                 "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                 "kernels_ms_per_step": {k: v[0] / args.steps for k, v in kern.items()},

@@ -445,6 +445,24 @@ int viscache_kv4_dequantize(const vc_batch* batch, const vc_params* p, const uin
 int viscache_set_kernel_path(int path);
 
 /*
+ * viscache_test_inject_wait -- test support for the failure detection of the
+ * tensor-core kernels (not a step of the pass).  For every later launch of
+ * a kernel named in kernel_mask, one consumer warp first waits on an
+ * mbarrier that nothing ever completes ("a flag that nothing sets"), bounded
+ * like every wait of these kernels but with a short limit (~10^5 SM clocks).
+ * When the wait gives up the kernel records VC_ERR_DEVICE_TIMEOUT in the
+ * status word and then does its normal work (its own barriers and copies are
+ * not touched), so the launch ends, the context stays usable, and the
+ * caller's prunekv_get_status / prunekv_score_static_status reads the error.
+ * kernel_mask 0 (the default) turns it off.  Process-wide; not thread-safe
+ * against concurrent calls.  Errors: VC_ERR_INVALID_ARG for unknown bits.
+ */
+#define VC_TEST_WAIT_SCORE_LSE    1  /* score_lse_tc: the row log-sum-exp pass */
+#define VC_TEST_WAIT_SCORE_COLSUM 2  /* score_colsum_tc: the column-sum pass */
+#define VC_TEST_WAIT_FUSE         4  /* fuse_v_tc: the value fusion */
+int viscache_test_inject_wait(int kernel_mask);
+
+/*
  * viscache_device_accessible -- 1 if the current device can read `ptr`
  * directly (device memory, managed memory, or host memory mapped into the
  * device's address space, e.g. pinned with cudaHostAlloc under unified

@@ -20,6 +20,8 @@ constexpr size_t kAlign = 256;
 
 // Kernel path: VC_PATH_AUTO uses the tcgen05 score kernels for bf16, d = 128.
 std::atomic<int> g_path{VC_PATH_AUTO};
+// Test support: kernels whose next launches add one wait that must give up.
+std::atomic<int> g_test_wait{0};
 
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
@@ -280,6 +282,7 @@ struct Layout {
     s.n_req = n_req;
     s.rank_mode = rank_mode;
     s.scale_log2 = scale * kLog2e;
+    s.test_wait = g_test_wait.load();
     return s;
   }
 };
@@ -553,6 +556,13 @@ int viscache_device_accessible(const void* ptr) {
   if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return 1;
   if (a.type == cudaMemoryTypeHost) return a.devicePointer == ptr ? 1 : 0;
   return 0;
+}
+
+int viscache_test_inject_wait(int kernel_mask) {
+  if (kernel_mask < 0 || kernel_mask > (VC_TEST_WAIT_SCORE_LSE | VC_TEST_WAIT_SCORE_COLSUM | VC_TEST_WAIT_FUSE))
+    return VC_ERR_INVALID_ARG;
+  g_test_wait.store(kernel_mask);
+  return VC_OK;
 }
 
 int viscache_set_kernel_path(int path) {

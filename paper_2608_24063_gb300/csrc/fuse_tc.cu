@@ -136,6 +136,7 @@ struct FSmem {
   uint64_t p_full[2];                  // even CTA: all 16 softmax warps wrote P(j), buffer j % 2
   uint64_t o_done;                     // both: O(j) is done (phase j)
   uint64_t mma_done;                   // both: every MMA of the pair is done (one phase)
+  uint64_t never;                      // test support: never completes
   uint32_t tmem_base;
   int abort;
 };
@@ -204,6 +205,7 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     mbar_init(&sm.p_full[1], 16);
     mbar_init(&sm.o_done, 1);
     mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.never, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -285,6 +287,10 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
     mma_commit_pair(&sm.mma_done, 3);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
+    if ((sh.test_wait & VC_TEST_WAIT_FUSE) && warp == 0) {
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      __syncwarp();
+    }
     // ---- softmax over the drop set and epilogue: one kept row per TMEM lane
     const int q4 = warp & 3;                          // lane quadrant
     const int hf = warp >> 2;                         // column half

@@ -114,6 +114,7 @@ struct P1Smem {
   uint64_t tm_full[2];                      // both: the slot's logits are ready
   uint64_t tm_empty[2];                     // even CTA: the slot's 8 consumer warps copied it out
   uint64_t mma_done;
+  uint64_t never;                           // test support: never completes
   uint32_t tmem_base;
   int abort;
 };
@@ -149,6 +150,7 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     for (int i = 0; i < kStagesPair; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
     for (int i = 0; i < 2; ++i) { mbar_init(&sm.tm_full[i], 1); mbar_init(&sm.tm_empty[i], 8); }
     mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.never, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -210,6 +212,10 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     mma_commit_pair(&sm.mma_done, 1);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
+    if ((sh.test_wait & VC_TEST_WAIT_SCORE_LSE) && warp == 0) {
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      __syncwarp();
+    }
     // ---- row statistics: one thread per row (= TMEM lane).  Warpgroup wg
     // takes the tiles i with i % 2 == wg (TMEM slot wg), all 256 columns in
     // two halves, so the two warpgroups on a sub-partition run a tile apart
@@ -431,6 +437,7 @@ struct P2Smem {
   uint64_t tm_full[2];                        // both: the slot's logits are ready
   uint64_t tm_empty[2];                       // even CTA: the slot's 8 consumer warps copied it out
   uint64_t mma_done;
+  uint64_t never;                             // test support: never completes
   uint32_t tmem_base;
   int abort;
 };
@@ -466,6 +473,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
       mbar_init(&sm.q_empty[i], 1 + 4);   // MMA commit + the stage's 4 consumer warps of this CTA
     }
     mbar_init(&sm.mma_done, 1);
+    mbar_init(&sm.never, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -546,6 +554,10 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     mma_commit_pair(&sm.mma_done, 1);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
+    if ((sh.test_wait & VC_TEST_WAIT_SCORE_COLSUM) && warp == 0) {
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      __syncwarp();
+    }
     // ---- column sums: one thread per key (= TMEM lane)
     const int wg = warp >> 2;
     const int key = ((warp & 3) << 5) + lane;

@@ -75,6 +75,23 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// Wait bounded by `limit` SM clocks (checked on every try); false on give-up.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, long long limit) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > limit) return false;
+  return true;
+}
+
+// Test support (Shape::test_wait): the calling lane waits on `never`, an
+// mbarrier initialised with one pending arrival that nothing ever makes, so
+// the bounded wait always gives up; the caller then records the timeout.
+constexpr long long kTestWaitCycles = 100000;
+
+__device__ __forceinline__ bool injected_wait_gives_up(uint64_t* never) {
+  return !mbar_wait_for(never, 0, kTestWaitCycles);
+}
+
 // ---------------------------------------------------------------------------
 // TMA
 

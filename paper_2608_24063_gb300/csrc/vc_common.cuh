@@ -44,6 +44,7 @@ struct Shape {
   int32_t n_req;
   int32_t rank_mode;
   float scale_log2;          // logit scale * log2(e)
+  int32_t test_wait;         // VC_TEST_WAIT_* bits (test support, normally 0)
 };
 
 struct Tables {              // device pointers into the workspace

@@ -29,6 +29,7 @@ VC_RANK_SHARED, VC_RANK_PER_LAYER = 0, 1
 VC_SCHED_PARABOLA, VC_SCHED_FIXED, VC_SCHED_ARITHMETIC, VC_SCHED_GEOMETRIC = 0, 1, 2, 3
 VC_DROP_SURVIVORS, VC_DROP_ALL = 0, 1
 VC_PATH_AUTO, VC_PATH_SIMT = 0, 1
+VC_TEST_WAIT_SCORE_LSE, VC_TEST_WAIT_SCORE_COLSUM, VC_TEST_WAIT_FUSE = 1, 2, 4
 
 _ERR_NAMES = {1: "VC_ERR_INVALID_ARG", 2: "VC_ERR_INFEASIBLE", 3: "VC_ERR_WORKSPACE",
               4: "VC_ERR_CUDA", 5: "VC_ERR_DEVICE_TIMEOUT", 6: "VC_ERR_UNSUPPORTED",
@@ -39,7 +40,7 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
             "viscache_profile_read", "prunekv_score_static", "prunekv_score_static_capacity",
-            "prunekv_score_static_status", "viscache_set_kernel_path",
+            "prunekv_score_static_status", "viscache_set_kernel_path", "viscache_test_inject_wait",
             "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_sizes", "viscache_scout_mmr",
             "viscache_decode_workspace_size", "viscache_decode_attention",
             "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize",
@@ -121,6 +122,7 @@ def lib() -> ctypes.CDLL:
         L.viscache_version.restype = ctypes.c_char_p
         L.viscache_profile_enable.argtypes = [i32]
         L.viscache_set_kernel_path.argtypes = [i32]
+        L.viscache_test_inject_wait.argtypes = [i32]
         L.viscache_device_accessible.argtypes = [vp]
         L.viscache_profile_read.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(ctypes.c_float),
                                             pi32, i32]
@@ -483,6 +485,11 @@ def viscache_kv4_dequantize(batch: Batch, params: vc_params, K_codes: torch.Tens
 def viscache_set_kernel_path(path: int) -> None:
     """VC_PATH_AUTO (tensor cores for bf16, d=128) or VC_PATH_SIMT (CUDA cores everywhere)."""
     _check("viscache_set_kernel_path", lib().viscache_set_kernel_path(path))
+
+
+def viscache_test_inject_wait(kernel_mask: int) -> None:
+    """Test support: the named tensor-core kernels add one wait that gives up (0 = off)."""
+    _check("viscache_test_inject_wait", lib().viscache_test_inject_wait(kernel_mask))
 
 
 def viscache_profile_enable(on: bool) -> None:

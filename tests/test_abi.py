@@ -243,3 +243,9 @@ def test_scout_sizes_match_oracle_keyframe_count():
     assert vc.lib().viscache_scout_sizes(1, one, 5, 4, out) == vc.VC_ERR_INVALID_ARG
     assert vc.lib().viscache_scout_sizes(1, (ctypes.c_int32 * 1)(0), 3, 4, out) == vc.VC_ERR_INVALID_ARG
     assert vc.lib().viscache_scout_sizes(1, one, 3, 4, None) == vc.VC_ERR_INVALID_ARG
+
+
+def test_test_wait_switch_rejects_unknown_bits():
+    assert vc.lib().viscache_test_inject_wait(8) == vc.VC_ERR_INVALID_ARG
+    assert vc.lib().viscache_test_inject_wait(-1) == vc.VC_ERR_INVALID_ARG
+    assert vc.lib().viscache_test_inject_wait(0) == vc.VC_OK

@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true", help="time direct launches instead of a CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sustain-seconds", type=float, default=1.5,
+                    help="repeat the K-step window for this long under the clock sampler (0: only the headline window)")
     ap.add_argument("--schedule", choices=list(SCHEDULES), default="parabola",
                     help="layer-budget schedule (the paper's ablation axes); parabola is the method")
     ap.add_argument("--stage", choices=["prunekv", "scout", "decode", "quant"], default="prunekv",
@@ -833,7 +835,7 @@ def main():
     # headline stays the first window of exactly K steps
     windows = []
     if args.steps > 0:
-        n_more = max(0, min(2000, int(math.ceil(1500.0 / max(ms, 1e-3))) - 1))
+        n_more = max(0, min(2000, int(math.ceil(args.sustain_seconds * 1e3 / max(ms, 1e-3))) - 1))
         ea = [torch.cuda.Event(enable_timing=True) for _ in range(n_more + 1)]
         for i in range(n_more):
             ea[i].record(st)

@@ -5,16 +5,18 @@
 //   kept key rows go to K_out (bit-exact), and the survivors' value rows --
 //   kept then dropped, each list in ascending position -- are compacted into a
 //   dense workspace slab Vs, so the fusion can stream them with TMA.
-// fuse_v_tc_kernel: one CTA pair per (request, layer, KV head, 256 kept rows):
+// fuse_v_tcp_kernel: persistent CTA pairs, each taking a share of the units
+//   (request, layer, KV head, 256 kept rows) in turn:
 //   O = softmax_row(V_k V_d^T / tau) V_d online over tiles of 128 dropped rows,
 //   V_out = mu V_k + (1 - mu) O, on 2-SM tcgen05.mma with fp32 accumulators in
 //   tensor memory; the numerators P go from the softmax warps to the second
-//   product through tensor memory.  Warp roles (320 threads, two CTAs per SM):
-//   warps 0-7 softmax and epilogue, warp 8 TMA and the tensor-memory
-//   allocation, one thread of warp 9 (even CTA) the MMAs.  Every wait is
-//   bounded (tc_common.cuh).
+//   product through tensor memory.  Warp roles (448 threads, one CTA per SM):
+//   warps 0-7 softmax, warp 8 TMA and the tensor-memory allocation, one
+//   thread of warp 9 (even CTA) the MMAs, warps 10-13 the epilogue.  Every
+//   wait is bounded (tc_common.cuh).
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "kernels.h"
@@ -86,60 +88,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// fusion on CTA pairs
-//
-// A pair owns 256 kept rows of one (request, layer, KV head) (CTA r: rows
-// r*128 ... r*128+127, one per TMEM lane) and streams the dropped rows in
-// tiles of 64.  Per tile j the even CTA issues
-//   S(j) = V_k V_d(j)^T  2-SM MMA, M = 256, N = 64 dropped rows (CTA r stages
-//                        dropped rows r*32 ... r*32+31, K-major),
-//   O += P(j) V_d(j)     2-SM MMA, M = 256, N = 128 value columns, K = 64 (CTA
-//                        r stages columns r*64 ... of all 64 dropped rows,
-//                        MN-major), A = P read from tensor memory,
-// in the order S(0), S(1), [P(0)] O(0), S(2), [P(1)] O(1), ...: S is double
-// buffered, so S(j+1) is computed while the softmax works on tile j.  P(j) is
-// written in bf16 over the first half of each softmax warp's own S(j)
-// columns; S(j+2) reuses the buffer only after O(j) (issued before it) has
-// read P(j).  Two pairs run per TPC, so one pair's prologue and epilogue
-// overlap the other's work.
-//
-// Tensor memory per CTA (256 columns): O in [0, 128), S/P buffer b in
-// [128 + 64b, 192 + 64b).  Softmax: warps w and w+4 share the TMEM lanes of
-// warp w % 4; warp w takes S columns 0-31 (dropped rows 0-31 of the tile), warp
-// w+4 columns 32-63.  They agree on the row's reference maximum through shared
-// memory each tile; the maximum is raised (and O rescaled in tensor memory,
-// after O(j-1) is done) only when a tile exceeds it by more than 2^8.
-
-constexpr int kThreads = 320;
-constexpr int kProducerWarp = 8, kMmaWarp = 9;
-constexpr uint32_t kTile = 128;                  // kept rows per CTA
-constexpr uint32_t kKB = kTile * 128;            // 128 rows x 128 bytes
-constexpr uint32_t kDTile = 64;                  // dropped rows per tile (both CTAs)
-constexpr uint32_t kDHalfKB = 32 * 128;          // 32 rows x 128 bytes
-constexpr uint32_t kDKB = kDTile * 128;          // 64 rows x 128 bytes
-constexpr int kVdStages = 4;
-constexpr uint32_t kTmemCols = 256;              // O: [0,128), S/P buffers: [128,192), [192,256)
-constexpr uint32_t kSCol = 128;
-constexpr float kRescaleLog2 = 8.f;
-
-struct FSmem {
-  uint8_t vk[2][kKB];                  // this CTA's 128 kept rows [K-block]: A of S = V_k V_d^T
-  uint8_t vdo[kVdStages][kDKB];        // all 64 dropped rows, this CTA's 64 columns: B of O += P V_d
-  uint8_t vds[kVdStages][2][kDHalfKB]; // this CTA's 32 dropped rows [stage][K-block]: B of S
-  float xmax[2][4][2][32];             // [tile & 1][lane quadrant][column half][lane]: tile maxima
-  float lsum[2][4][32];                // [column half][lane quadrant][lane]: partial row sums
-  uint64_t vk_own;                     // this CTA's kept rows landed
-  uint64_t vk_pair;                    // even CTA: both CTAs' kept rows landed (2 arrivals)
-  uint64_t vd_full[kVdStages];         // even CTA: both CTAs' dropped tiles landed
-  uint64_t vd_empty[kVdStages];        // both: the MMAs reading the stage are done
-  uint64_t s_full[2];                  // both: S(j) is in S/P buffer j % 2
-  uint64_t p_full[2];                  // even CTA: all 16 softmax warps wrote P(j), buffer j % 2
-  uint64_t o_done;                     // both: O(j) is done (phase j)
-  uint64_t mma_done;                   // both: every MMA of the pair is done (one phase)
-  uint64_t never;                      // test support: never completes
-  uint32_t tmem_base;
-  int abort;
-};
+// shared helpers of the fusion
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   const uint32_t a = smem_u32(p);
@@ -167,43 +116,133 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 2)
-fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_constant__ CUtensorMap tmRows64,
-                 const __grid_constant__ CUtensorMap tmRows32, Shape sh, Tables tb, float mu, float c2,
-                 __nv_bfloat16* __restrict__ V_out) {
+// ---------------------------------------------------------------------------
+// persistent fusion: one CTA pair per TPC for the whole launch
+//
+// Same arithmetic as fuse_v_tc_kernel, organised so that nothing waits at a
+// unit boundary.  The launch holds as many pairs as fit at once (one CTA per
+// SM: 512 tensor-memory columns and ~214 KB of shared memory each); pair p
+// takes the units p, p + P, p + 2P, ... of the list ordered longest first.
+// Tensor memory per CTA: O[0] [0,128), O[1] [128,256) -- unit k accumulates
+// in O[k % 2] -- and S[0] [256,384), S[1] [384,512) -- dropped tile t (counted
+// over all of the pair's units) lands in S[t % 2], P(t) over the first half of
+// each softmax warp's 64 columns.  Tiles hold 128 dropped rows (N = 128 for
+// S, K = 128 for O: 16 MMAs and 2-3 commits per tile).  The issue order is
+// S(t), O(t-1), so S(t) runs while the softmax works on tile t-1.
+//
+// Warps: 0-7 softmax (as in fuse_v_tc_kernel, 64 columns each), 8 the
+// producer (lane 0 issues the TMA loads: the unit's kept rows into vk[k % 2],
+// then its dropped tiles into a 3-stage ring; lane 1 tells the even CTA when
+// this CTA's kept rows of each unit have landed), 9 the MMA issuer (even
+// CTA), 10-13 the epilogue: once O[k % 2] is final it reads O, the row sums
+// and V_k, writes mu V_k + (1 - mu) O / lsum in bf16 through a staging buffer,
+// and frees O[k % 2] and vk[k % 2] -- while the MMAs and the softmax of unit
+// k + 1 go on.
+//
+// Every barrier completes once per unit (or per tile) and no waiter can fall
+// two phases behind: the loader refills vk[b] only after the epilogue freed it,
+// the MMA issuer overwrites O[b] (first O of a unit) only after the epilogue
+// freed it, and the softmax writes a unit's row sums only after the epilogue
+// read those of the unit two before.  A unit with no dropped rows still runs
+// through every handshake (the issuer commits its O barrier without MMAs), so
+// phases stay aligned with unit indices.  All waits are bounded.
+
+namespace pf {
+
+constexpr int kProducerWarp = 8, kMmaWarp = 9, kEpiWarp0 = 10, kEpiWarps = 4;
+constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);   // 448
+constexpr uint32_t kTile = 128;                  // kept rows per CTA
+constexpr uint32_t kKB = kTile * 128;            // 128 rows x 128 bytes
+constexpr uint32_t kDTile = 128;                 // dropped rows per tile (both CTAs)
+constexpr uint32_t kDHalf = kDTile / 2;          // dropped rows staged per CTA for S
+constexpr uint32_t kDHalfKB = kDHalf * 128;      // 64 rows x 128 bytes
+constexpr uint32_t kDKB = kDTile * 128;          // 128 rows x 128 bytes
+constexpr int kStages = 3;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kSCol = 256;
+constexpr int kMaxUnits = 512;                   // units per pair (descriptor table)
+constexpr float kRescaleLog2 = 8.f;
+
+struct Unit {              // one unit as this CTA sees it
+  int32_t vk_row;          // Vs row of this CTA's first kept row
+  int32_t vd_row;          // Vs row of the (layer, KV head)'s first dropped row
+  int32_t D;               // dropped rows
+  int32_t rows;            // kept rows of this CTA (0..128)
+  int64_t orow;            // V_out row of this CTA's first kept row
+  int64_t pad;
+};
+
+struct Smem {
+  uint8_t vk[2][2][kKB];               // kept rows of unit k in vk[k % 2] [K-block]
+  uint8_t vdo[kStages][kDKB];          // dropped tile: all 128 rows, this CTA's 64 columns (B of O)
+  uint8_t vds[kStages][2][kDHalfKB];   // dropped tile: this CTA's 64 rows [K-block] (B of S)
+  uint8_t stg[kTile * 256];            // epilogue staging, 128 rows x 256 bytes
+  Unit unit[kMaxUnits];
+  float xmax[2][4][2][32];             // [tile & 1][lane quadrant][column half][lane]
+  float lsum[2][4][2][32];             // [unit & 1][lane quadrant][column half][lane]
+  uint64_t vk_full[2];                 // own kept rows landed (1 arrival + bytes)
+  uint64_t vk_pair[2];                 // even CTA: both CTAs' kept rows landed (2)
+  uint64_t vk_empty[2];                // own: the epilogue read vk[b] (4 warps)
+  uint64_t vd_full[kStages];           // even CTA: both CTAs' dropped tiles landed
+  uint64_t vd_empty[kStages];          // both: the O product reading the stage is done
+  uint64_t s_full[2];                  // both: S(t) in S[t % 2]
+  uint64_t p_full[2];                  // even CTA: the 16 softmax warps wrote P(t)
+  uint64_t o_full[2];                  // both: the unit's O[b] is final
+  uint64_t o_empty[2];                 // even CTA: the 8 epilogue warps read O[b]
+  uint64_t lsum_full[2];               // own: the 8 softmax warps wrote the unit's row sums
+  uint64_t lsum_empty[2];              // own: the 4 epilogue warps read them
+  uint64_t mma_done;                   // both: every MMA of the pair is done
+  uint64_t never;                      // test support: never completes
+  uint32_t tmem_base;
+  int abort;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_constant__ CUtensorMap tmRows64,
+                  Shape sh, Tables tb, int units, int o_lo, int o_cnt, float mu, float c2,
+                  __nv_bfloat16* __restrict__ V_out) {
   extern __shared__ uint8_t smem_raw[];
-  FSmem& sm = *reinterpret_cast<FSmem*>(align1024(smem_raw));
+  Smem& sm = *reinterpret_cast<Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
-  // units in reverse order: later layers have fewer kept and more dropped
-  // rows, so their units are the longest; starting them first leaves the
-  // short units of the first layers to fill the last wave
-  const int unit = (int)(gridDim.x >> 1) - 1 - (int)(blockIdx.x >> 1);
+  const int pair = (int)(blockIdx.x >> 1), npairs = (int)(gridDim.x >> 1);
+  // this launch covers positions [o_lo, o_lo + o_cnt) of the longest-first unit
+  // order (position o is unit units-1-o); pair p takes o_lo + p, o_lo + p + P, ...
+  const int nunits = min(kMaxUnits, (o_cnt - pair + npairs - 1) / npairs);
 
-  const int rl = upper_index_warp(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
-  const int r = rl / sh.L;
-  const Req rq = tb.req[r];
-  const Layer ly = tb.layer[rl];
-  const int ktiles = (ly.B + 2 * (int)kTile - 1) / (2 * (int)kTile);
-  const int u = unit - tb.unit0_fuse_tc[rl];
-  const int g = u / ktiles;
-  const int r0 = (u % ktiles) * 2 * (int)kTile + (int)rank * (int)kTile;   // this CTA's first kept row
-  const int rows = max(0, min((int)kTile, ly.B - r0));                    // kept rows of this CTA
-  const int D = ly.D;
-  const int nt = (D + (int)kDTile - 1) / (int)kDTile;
-  // rows of this (layer, KV head) in Vs: B kept, then D dropped
-  const int vs0 = (int)(rq.vs_row0 + (int64_t)sh.Hkv * (ly.P + ly.Qd) + (int64_t)g * (ly.B + D));
-  const int64_t orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
-
+  // this pair's unit descriptors
+  for (int i = threadIdx.x; i < nunits; i += kThreads) {
+    const int unit = units - 1 - (o_lo + pair + i * npairs);
+    const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
+    const Req rq = tb.req[rl / sh.L];
+    const Layer ly = tb.layer[rl];
+    const int ktiles = (ly.B + 2 * (int)kTile - 1) / (2 * (int)kTile);
+    const int u = unit - tb.unit0_fuse_tc[rl];
+    const int g = u / ktiles;
+    const int r0 = (u % ktiles) * 2 * (int)kTile + (int)rank * (int)kTile;
+    const int vs0 = (int)(rq.vs_row0 + (int64_t)sh.Hkv * (ly.P + ly.Qd) + (int64_t)g * (ly.B + ly.D));
+    Unit d;
+    d.vk_row = vs0 + r0;
+    d.vd_row = vs0 + ly.B;
+    d.D = ly.D;
+    d.rows = max(0, min((int)kTile, ly.B - r0));
+    d.orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
+    d.pad = 0;
+    sm.unit[i] = d;
+  }
   if (threadIdx.x == 0) {
-    mbar_init(&sm.vk_own, 1);
-    mbar_init(&sm.vk_pair, 2);
-    for (int i = 0; i < kVdStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
-    mbar_init(&sm.s_full[0], 1);
-    mbar_init(&sm.s_full[1], 1);
-    mbar_init(&sm.p_full[0], 16);
-    mbar_init(&sm.p_full[1], 16);
-    mbar_init(&sm.o_done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.vk_full[b], 1);
+      mbar_init(&sm.vk_pair[b], 2);
+      mbar_init(&sm.vk_empty[b], kEpiWarps);
+      mbar_init(&sm.s_full[b], 1);
+      mbar_init(&sm.p_full[b], 16);
+      mbar_init(&sm.o_full[b], 1);
+      mbar_init(&sm.o_empty[b], 2 * kEpiWarps);
+      mbar_init(&sm.lsum_full[b], 8);
+      mbar_init(&sm.lsum_empty[b], kEpiWarps);
+    }
+    for (int i = 0; i < kStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
     mbar_init(&sm.mma_done, 1);
     mbar_init(&sm.never, 1);
     sm.abort = 0;
@@ -215,75 +254,101 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
   }
   __syncwarp();
   tc_fence_before();
-  cluster_sync();
+  cluster_sync();                  // descriptors, barriers of both CTAs, TMEM
   tc_fence_after();
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
 
   if (warp == kProducerWarp && lane == 0) {
-    // ---- TMA producer (both CTAs)
+    // ---- TMA loader (both CTAs)
     prefetch_tmap(&tmRows128);
     prefetch_tmap(&tmRows64);
-    prefetch_tmap(&tmRows32);
-    mbar_arrive_expect_tx(&sm.vk_own, 2 * kKB);
-    for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.vk[kb], &tmRows128, kb * 64, vs0 + r0, &sm.vk_own);
-    int issued = 0;
-    for (int j = 0; j < nt; ++j) {
-      if (j == kVdStages) {
-        // the ring is full: own kept rows landed -> tell the even CTA, whose
-        // MMAs read them (and must run before any stage frees up)
-        if (!mbar_wait(&sm.vk_own, 0, abort)) break;
-        mbar_arrive_cluster(map_to_rank(smem_u32(&sm.vk_pair), 0));
+    int t = 0, kl = 0;
+    bool ok = true;
+    for (int k = 0; ok && k < nunits; ++k) {
+      const Unit d = sm.unit[k];
+      const int b = k & 1;
+      if (!mbar_wait(&sm.vk_empty[b], ((k >> 1) & 1) ^ 1, abort)) break;
+      mbar_arrive_expect_tx(&sm.vk_full[b], 2 * kKB);
+      for (int kb = 0; kb < 2; ++kb) tma_load_2d(sm.vk[b][kb], &tmRows128, kb * 64, d.vk_row, &sm.vk_full[b]);
+      ++kl;
+      const int nt = (d.D + (int)kDTile - 1) / (int)kDTile;
+      for (int j = 0; j < nt; ++j) {
+        const int st = t % kStages;
+        if (!mbar_wait(&sm.vd_empty[st], ((t / kStages) & 1) ^ 1, abort)) { ok = false; break; }
+        if (rank == 0) mbar_arrive_expect_tx(&sm.vd_full[st], 2 * (2 * kDHalfKB + kDKB));
+        const uint32_t full0 = map_to_rank(smem_u32(&sm.vd_full[st]), 0);
+        const int y = d.vd_row + j * (int)kDTile;
+        tma_load_2d_pair(sm.vds[st][0], &tmRows64, 0, y + (int)rank * (int)kDHalf, full0);
+        tma_load_2d_pair(sm.vds[st][1], &tmRows64, 64, y + (int)rank * (int)kDHalf, full0);
+        tma_load_2d_pair(sm.vdo[st], &tmRows128, (int)rank * 64, y, full0);
+        ++t;
       }
-      const int st = j % kVdStages;
-      if (!mbar_wait(&sm.vd_empty[st], ((j / kVdStages) & 1) ^ 1, abort)) break;
-      if (rank == 0) mbar_arrive_expect_tx(&sm.vd_full[st], 2 * (2 * kDHalfKB + kDKB));
-      const uint32_t full0 = map_to_rank(smem_u32(&sm.vd_full[st]), 0);
-      const int y = vs0 + ly.B + j * (int)kDTile;
-      tma_load_2d_pair(sm.vds[st][0], &tmRows32, 0, y + (int)rank * 32, full0);
-      tma_load_2d_pair(sm.vds[st][1], &tmRows32, 64, y + (int)rank * 32, full0);
-      tma_load_2d_pair(sm.vdo[st], &tmRows64, (int)rank * 64, y, full0);
-      ++issued;
     }
-    if (nt <= kVdStages && mbar_wait(&sm.vk_own, 0, abort))
-      mbar_arrive_cluster(map_to_rank(smem_u32(&sm.vk_pair), 0));
+    // every copy this CTA started has landed before the pair may leave
+    for (int i = max(0, kl - 2); i < kl; ++i) drain_wait(&sm.vk_full[i & 1], (i >> 1) & 1);
     if (rank == 0)
-      for (int i = max(0, issued - kVdStages); i < issued; ++i)
-        drain_wait(&sm.vd_full[i % kVdStages], (i / kVdStages) & 1);
-  } else if (warp == kMmaWarp && lane == 0 && rank == 0 && nt > 0) {
-    // ---- MMA issuer (even CTA): S(0), S(1), O(0), S(2), O(1), ...
+      for (int i = max(0, t - kStages); i < t; ++i) drain_wait(&sm.vd_full[i % kStages], (i / kStages) & 1);
+  } else if (warp == kProducerWarp && lane == 1) {
+    // ---- kept-rows relay: this CTA's kept rows of unit k landed -> even CTA
+    const uint32_t pair0 = map_to_rank(smem_u32(&sm.vk_pair[0]), 0);
+    const uint32_t pair1 = map_to_rank(smem_u32(&sm.vk_pair[1]), 0);
+    for (int k = 0; k < nunits; ++k) {
+      if (!mbar_wait(&sm.vk_full[k & 1], (k >> 1) & 1, abort)) break;
+      mbar_arrive_cluster((k & 1) ? pair1 : pair0);
+    }
+  } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
+    // ---- MMA issuer (even CTA): S(t), then O(t-1)
     const uint32_t id_s = idesc_bf16_f32(2 * kTile, kDTile);
     const uint32_t id_o = idesc_bf16_f32_bmn(2 * kTile, kTile);
-    bool ok = mbar_wait(&sm.vk_pair, 0, abort);
-    for (int j = 0; ok && j <= nt; ++j) {
-      if (j < nt) {
-        // S(j) into buffer j % 2 (its previous user O(j-2) was issued before)
-        const int st = j % kVdStages;
-        if (!mbar_wait(&sm.vd_full[st], (j / kVdStages) & 1, abort)) break;
+    struct Pend { int t, st, k, b; bool first, last; };
+    Pend pv{0, 0, 0, 0, false, false};
+    bool have = false, ok = true;
+    // O(pv.t) += P(pv.t) V_d(pv.t); frees the stage, and finishes O[b] on a unit's last tile
+    auto issue_o = [&](const Pend& q) -> bool {
+      if (q.first && !mbar_wait(&sm.o_empty[q.b], ((q.k >> 1) & 1) ^ 1, abort)) return false;
+      if (!mbar_wait(&sm.p_full[q.t & 1], (q.t >> 1) & 1, abort)) return false;
+      tc_fence_after();
+      const uint32_t p_tm = tbase + kSCol + (uint32_t)(q.t & 1) * kDTile;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        mma_bf16_pair_ta(tbase + (uint32_t)q.b * kTile, p_tm + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
+                         desc_sw128_mn(smem_u32(sm.vdo[q.st]) + kk * 2048, kDKB), id_o,
+                         (!q.first || kk > 0) ? 1u : 0u);
+      mma_commit_pair(&sm.vd_empty[q.st], 3);
+      if (q.last) mma_commit_pair(&sm.o_full[q.b], 3);
+      return true;
+    };
+    int t = 0;
+    for (int k = 0; ok && k < nunits; ++k) {
+      const Unit d = sm.unit[k];
+      const int b = k & 1;
+      const int nt = (d.D + (int)kDTile - 1) / (int)kDTile;
+      if (!mbar_wait(&sm.vk_pair[b], (k >> 1) & 1, abort)) { ok = false; break; }
+      if (nt == 0) {
+        // nothing dropped: V_out = V_k; keep the O[b] handshake in step
+        if (have) { ok = issue_o(pv); have = false; if (!ok) break; }
+        if (!mbar_wait(&sm.o_empty[b], ((k >> 1) & 1) ^ 1, abort)) { ok = false; break; }
+        mma_commit_pair(&sm.o_full[b], 3);
+        continue;
+      }
+      for (int j = 0; j < nt; ++j, ++t) {
+        const int st = t % kStages;
+        if (!mbar_wait(&sm.vd_full[st], (t / kStages) & 1, abort)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t s_tm = tbase + kSCol + (uint32_t)(j & 1) * kDTile;
+        const uint32_t s_tm = tbase + kSCol + (uint32_t)(t & 1) * kDTile;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          mma_bf16_pair(s_tm, desc_sw128(smem_u32(sm.vk[kk >> 2]) + (kk & 3) * 32),
+          mma_bf16_pair(s_tm, desc_sw128(smem_u32(sm.vk[b][kk >> 2]) + (kk & 3) * 32),
                         desc_sw128(smem_u32(sm.vds[st][kk >> 2]) + (kk & 3) * 32), id_s, kk ? 1u : 0u);
-        mma_commit_pair(&sm.s_full[j & 1], 3);
-      }
-      if (j >= 1) {
-        // O += P(j-1) V_d(j-1), once the softmax has written P(j-1)
-        const int jp = j - 1, st = jp % kVdStages;
-        if (!mbar_wait(&sm.p_full[jp & 1], (jp >> 1) & 1, abort)) break;
-        tc_fence_after();
-        const uint32_t p_tm = tbase + kSCol + (uint32_t)(jp & 1) * kDTile;
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          mma_bf16_pair_ta(tbase, p_tm + (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8),
-                           desc_sw128_mn(smem_u32(sm.vdo[st]) + kk * 2048, kDKB), id_o,
-                           (jp > 0 || kk > 0) ? 1u : 0u);
-        mma_commit_pair(&sm.vd_empty[st], 3);
-        mma_commit_pair(&sm.o_done, 3);
+        mma_commit_pair(&sm.s_full[t & 1], 3);
+        if (have && !issue_o(pv)) { ok = false; break; }
+        pv = Pend{t, st, k, b, j == 0, j == nt - 1};
+        have = true;
       }
     }
-    // always committed (also after a give-up), so the epilogue's wait ends
+    if (ok && have) issue_o(pv);
+    // always committed (also after a give-up), so every wait on it ends
     mma_commit_pair(&sm.mma_done, 3);
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
@@ -291,137 +356,152 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
       if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
       __syncwarp();
     }
-    // ---- softmax over the drop set and epilogue: one kept row per TMEM lane
-    const int q4 = warp & 3;                          // lane quadrant
-    const int hf = warp >> 2;                         // column half
-    const int row = (q4 << 5) + lane;                 // row within this CTA's 128
+    // ---- softmax over the drop set: one kept row per TMEM lane
+    const int q4 = warp & 3, hf = warp >> 2;
     const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
-    const uint32_t o_col = tbase + lane_off + (uint32_t)hf * 64;
-    float m = -INFINITY, lsum = 0.f;
+    int t = 0;
     bool ok = true;
-    for (int j = 0; j < nt; ++j) {
-      const int bsel = j & 1;
-      if (!warp_wait(&sm.s_full[bsel], (j >> 1) & 1, abort)) { ok = false; break; }
-      tc_fence_after();
-      // this warp's 32 columns of S(j)
-      const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)bsel * kDTile + (uint32_t)hf * 32;
-      float x[2][16];
-      {
-        uint32_t v[2][16];
-#pragma unroll
-        for (int p = 0; p < 2; ++p) tmem_ld16(s_col + p * 16, v[p]);
-        tmem_wait_only();
-#pragma unroll
-        for (int p = 0; p < 2; ++p) {
-          reg_fence(v[p]);
-#pragma unroll
-          for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
-        }
-      }
-      const int valid = min(32, D - j * (int)kDTile - hf * 32);
-      if (valid < 32) {                               // last tile: columns past D
-#pragma unroll
-        for (int p = 0; p < 2; ++p)
-#pragma unroll
-          for (int q = 0; q < 16; ++q)
-            if (p * 16 + q >= valid) x[p][q] = -INFINITY;
-      }
-      float a0 = fmaxf(x[0][0], x[0][1]), a1 = fmaxf(x[1][0], x[1][1]);
-#pragma unroll
-      for (int q = 2; q < 16; q += 2) {
-        a0 = fmax3(a0, x[0][q], x[0][q + 1]);
-        a1 = fmax3(a1, x[1][q], x[1][q + 1]);
-      }
-      // this row's tile maximum over both column halves
-      sm.xmax[bsel][q4][hf][lane] = fmaxf(a0, a1);
-      named_sync(1 + q4, 64);
-      const float tm = fmaxf(sm.xmax[bsel][q4][0][lane], sm.xmax[bsel][q4][1][lane]) * c2;
-      const bool raise = tm > m + kRescaleLog2;
-      const float m_new = raise ? tm : m;
-      const float corr = raise ? ex2(m - m_new) : 1.f;   // 0 on the first tile
-      lsum *= corr;
-      m = m_new;
-      // P = exp2(S * c2 - m) in bf16 over the first 16 of this warp's S columns
-      const float2 sc = make_float2(c2, c2), nm = make_float2(-m, -m);
-      float2 ls = make_float2(0.f, 0.f);
-      {
-        uint32_t w[16];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          const int c = 2 * q;
-          const float2 t = __ffma2_rn(make_float2(x[c >> 4][c & 15], x[c >> 4][(c & 15) + 1]), sc, nm);
-          const float2 e = make_float2(ex2(t.x), ex2(t.y));
-          ls = __fadd2_rn(ls, e);
-          w[q] = pack_bf16x2(e.x, e.y);
-        }
-        tmem_st16(s_col, w);
-      }
-      lsum += ls.x + ls.y;
-      if (__any_sync(0xffffffffu, raise && j > 0)) {
-        // rare: rescale this warp's 64 columns of O in tensor memory once
-        // O(j-1) is done (O(j) waits for P(j), so nothing else writes O).  The
-        // parity wait is unambiguous: s_full(j) was committed after O(j-2), so
-        // o_done is in phase j-1 or j here.
-        if (!warp_wait(&sm.o_done, (j - 1) & 1, abort)) { ok = false; break; }
+    for (int k = 0; ok && k < nunits; ++k) {
+      const Unit d = sm.unit[k];
+      const int b = k & 1;
+      const int nt = (d.D + (int)kDTile - 1) / (int)kDTile;
+      const uint32_t o_col = tbase + lane_off + (uint32_t)b * kTile + (uint32_t)hf * 64;
+      float m = -INFINITY, lsum = 0.f;
+      for (int j = 0; j < nt; ++j, ++t) {
+        const int bsel = t & 1;
+        if (!warp_wait(&sm.s_full[bsel], (t >> 1) & 1, abort)) { ok = false; break; }
         tc_fence_after();
-#pragma unroll 1
+        const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)bsel * kDTile + (uint32_t)hf * 64;
+        float x[4][16];
+        {
+          uint32_t v[4][16];
+#pragma unroll
+          for (int p = 0; p < 4; ++p) tmem_ld16(s_col + p * 16, v[p]);
+          tmem_wait_only();
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            reg_fence(v[p]);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) x[p][q] = __uint_as_float(v[p][q]);
+          }
+        }
+        const int valid = min(64, d.D - j * (int)kDTile - hf * 64);
+        if (valid < 64) {                             // last tile: columns past D
+#pragma unroll
+          for (int p = 0; p < 4; ++p)
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+              if (p * 16 + q >= valid) x[p][q] = -INFINITY;
+        }
+        float a[4];
+#pragma unroll
         for (int p = 0; p < 4; ++p) {
-          uint32_t v[16];
-          tmem_ld16(o_col + p * 16, v);
-          tmem_wait(v);
+          a[p] = fmaxf(x[p][0], x[p][1]);
 #pragma unroll
-          for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
-          tmem_st16(o_col + p * 16, v);
+          for (int q = 2; q < 16; q += 2) a[p] = fmax3(a[p], x[p][q], x[p][q + 1]);
         }
-      }
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&sm.p_full[bsel]), 0));
-    }
-    // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum, or V_k when nothing is dropped
-    sm.lsum[hf][q4][lane] = lsum;
-    const bool have_k = warp_wait(&sm.vk_own, 0, abort);
-    // O is final once every MMA of the pair is done.  (A parity wait on o_done
-    // for O(nt-1) would be ambiguous here: s_full(nt-1) only guarantees O(nt-3),
-    // and with O(nt-2) still running the barrier sits in a phase of the other
-    // parity, which that wait would take as complete.)
-    const bool have_o = have_k && ok && nt > 0 && warp_wait(&sm.mma_done, 0, abort);
-    __syncwarp();
-    named_sync(5, 256);
-    const float lt = sm.lsum[0][q4][lane] + sm.lsum[1][q4][lane];   // same order in both halves
-    if (have_o) tc_fence_after();
-    const float w_o = have_o ? (1.f - mu) / lt : 0.f;
-    const float w_k = have_o ? mu : 1.f;
-    // stage the 128 x 128 output tile in the (now idle) dropped-row buffers
-    // (vdo, 4 x 8 KB contiguous): row r at r * 256 bytes, 16-byte chunk c at
-    // slot c ^ (r & 15)
-    uint8_t* stage = &sm.vdo[0][0];
+        sm.xmax[bsel][q4][hf][lane] = fmaxf(fmaxf(a[0], a[1]), fmaxf(a[2], a[3]));
+        named_sync(1 + q4, 64);
+        const float tm = fmaxf(sm.xmax[bsel][q4][0][lane], sm.xmax[bsel][q4][1][lane]) * c2;
+        const bool raise = tm > m + kRescaleLog2;
+        const float m_new = raise ? tm : m;
+        const float corr = raise ? ex2(m - m_new) : 1.f;   // 0 on a unit's first tile
+        lsum *= corr;
+        m = m_new;
+        const float2 sc = make_float2(c2, c2), nm = make_float2(-m, -m);
+        float2 ls0 = make_float2(0.f, 0.f), ls1 = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          uint32_t w[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const int c = 32 * h + 2 * q;
+            const float2 tt = __ffma2_rn(make_float2(x[c >> 4][c & 15], x[c >> 4][(c & 15) + 1]), sc, nm);
+            const float2 e = make_float2(ex2(tt.x), ex2(tt.y));
+            if (q & 1) ls1 = __fadd2_rn(ls1, e);
+            else ls0 = __fadd2_rn(ls0, e);
+            w[q] = pack_bf16x2(e.x, e.y);
+          }
+          tmem_st16(s_col + h * 16, w);
+        }
+        const float2 ls = __fadd2_rn(ls0, ls1);
+        lsum += ls.x + ls.y;
+        if (__any_sync(0xffffffffu, raise && j > 0)) {
+          // rare: rescale this warp's 64 columns of O[b] once O(t-1) is done (its
+          // commit frees stage (t-1) % kStages); O(t) waits for P(t), below
+          const int tp = t - 1;
+          if (!warp_wait(&sm.vd_empty[tp % kStages], (tp / kStages) & 1, abort)) { ok = false; break; }
+          tc_fence_after();
 #pragma unroll 1
-    for (int hh = 0; hh < 2; ++hh) {                  // 32 of this warp's 64 columns at a time
-      float o[2][16];
-      if (have_o) {
-        uint32_t v[2][16];
+          for (int p = 0; p < 4; ++p) {
+            uint32_t v[16];
+            tmem_ld16(o_col + p * 16, v);
+            tmem_wait(v);
 #pragma unroll
-        for (int p = 0; p < 2; ++p) tmem_ld16(o_col + hh * 32 + p * 16, v[p]);
-        tmem_wait_only();
-#pragma unroll
-        for (int p = 0; p < 2; ++p) {
-          reg_fence(v[p]);
-#pragma unroll
-          for (int q = 0; q < 16; ++q) o[p][q] = __uint_as_float(v[p][q]);
+            for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
+            tmem_st16(o_col + p * 16, v);
+          }
         }
-      } else {
-#pragma unroll
-        for (int p = 0; p < 2; ++p)
-#pragma unroll
-          for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&sm.p_full[bsel]), 0));
       }
-      if (have_k) {
+      if (!ok) break;
+      // the unit's row sums, once the epilogue has read those of unit k - 2
+      if (!warp_wait(&sm.lsum_empty[b], ((k >> 1) & 1) ^ 1, abort)) break;
+      sm.lsum[b][q4][hf][lane] = lsum;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.lsum_full[b]);
+    }
+  } else if (warp >= kEpiWarp0) {
+    // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum (V_k when nothing is dropped)
+    const int q4 = warp & 3;                          // TMEM lane quadrant of this warp
+    const int row = (q4 << 5) + lane;
+    const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
+    const uint32_t o_empty0 = map_to_rank(smem_u32(&sm.o_empty[0]), 0);
+    const uint32_t o_empty1 = map_to_rank(smem_u32(&sm.o_empty[1]), 0);
+    const int te = (warp - kEpiWarp0) * 32 + lane;    // 0..127
+    for (int k = 0; k < nunits; ++k) {
+      const Unit d = sm.unit[k];
+      const int b = k & 1;
+      const uint32_t ph = (k >> 1) & 1;
+      if (!warp_wait(&sm.vk_full[b], ph, abort) || !warp_wait(&sm.lsum_full[b], ph, abort) ||
+          !warp_wait(&sm.o_full[b], ph, abort))
+        break;
+      tc_fence_after();
+      const bool have_o = d.D > 0;
+      const float lt = sm.lsum[b][q4][0][lane] + sm.lsum[b][q4][1][lane];   // same order as fuse_v_tc
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.lsum_empty[b]);
+      const float w_o = have_o ? (1.f - mu) / lt : 0.f;
+      const float w_k = have_o ? mu : 1.f;
+      const uint32_t o_col = tbase + lane_off + (uint32_t)b * kTile;
+#pragma unroll 1
+      for (int hh = 0; hh < 4; ++hh) {                // 32 output columns at a time
+        float o[2][16];
+        if (have_o) {
+          uint32_t v[2][16];
+#pragma unroll
+          for (int p = 0; p < 2; ++p) tmem_ld16(o_col + hh * 32 + p * 16, v[p]);
+          tmem_wait_only();
+#pragma unroll
+          for (int p = 0; p < 2; ++p) {
+            reg_fence(v[p]);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) o[p][q] = __uint_as_float(v[p][q]);
+          }
+        } else {
+#pragma unroll
+          for (int p = 0; p < 2; ++p)
+#pragma unroll
+            for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
+        }
+        const int kb = hh >> 1;
 #pragma unroll
         for (int c4 = 0; c4 < 4; ++c4) {
-          const int c8 = hh * 4 + c4;                 // 16-byte chunk within the K-block
-          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[hf][0] + swz(row, c8));
+          const int c8 = (hh & 1) * 4 + c4;             // 16-byte chunk within K-block kb
+          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[b][kb][0] + swz(row, c8));
           const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
           uint4 w;
           uint32_t* wp = &w.x;
@@ -429,25 +509,29 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
           for (int q = 0; q < 4; ++q) {
             const float2 kf = __bfloat1622float2(k2[q]);
             const float a = fmaf(w_k, kf.x, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q]);
-            const float b = fmaf(w_k, kf.y, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q + 1]);
-            wp[q] = pack_bf16x2(a, b);
+            const float bb = fmaf(w_k, kf.y, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q + 1]);
+            wp[q] = pack_bf16x2(a, bb);
           }
-          const int c = hf * 8 + c8;
-          *reinterpret_cast<uint4*>(stage + row * 256 + ((c ^ (row & 15)) << 4)) = w;
+          const int c = kb * 8 + c8;
+          *reinterpret_cast<uint4*>(&sm.stg[0] + row * 256 + ((c ^ (row & 15)) << 4)) = w;
         }
       }
-    }
-    named_sync(5, 256);
-    // coalesced copy-out: 16 threads per 256-byte row
-    const int t = threadIdx.x;                        // 0..255
-    if (have_k) {
-#pragma unroll 4
-      for (int i = 0; i < 8; ++i) {
-        const int rr = i * 16 + (t >> 4), c = t & 15;
-        if (rr < rows)
-          *reinterpret_cast<uint4*>(V_out + (orow + rr) * 128 + c * 8) =
-              *reinterpret_cast<const uint4*>(stage + rr * 256 + ((c ^ (rr & 15)) << 4));
+      // O[b] and vk[b] are read: free them
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive_cluster(b ? o_empty1 : o_empty0);
+        mbar_arrive(&sm.vk_empty[b]);
       }
+      named_sync(5, 32 * kEpiWarps);                 // staging complete
+#pragma unroll 4
+      for (int i = 0; i < 16; ++i) {                  // coalesced copy-out, 16 threads per row
+        const int rr = i * 8 + (te >> 4), c = te & 15;
+        if (rr < d.rows)
+          *reinterpret_cast<uint4*>(V_out + (d.orow + rr) * 128 + c * 8) =
+              *reinterpret_cast<const uint4*>(&sm.stg[0] + rr * 256 + ((c ^ (rr & 15)) << 4));
+      }
+      named_sync(5, 32 * kEpiWarps);                 // staging free for the next unit
     }
   }
   __syncwarp();
@@ -459,6 +543,8 @@ fuse_v_tc_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_con
   }
   if (threadIdx.x == 0 && sm.abort) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
 }
+
+}  // namespace pf
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -489,8 +575,33 @@ bool make_rows_map(CUtensorMap* m, const void* base, uint64_t rows, uint32_t box
 
 }  // namespace
 
-int fuse_rows_per_tile_tc() { return 2 * (int)kTile; }
+int fuse_rows_per_tile_tc() { return 2 * (int)pf::kTile; }
 int gather_rows_per_block() { return kGatherRows; }
+
+// CTA pairs of the persistent fusion that fit on the device at once.
+int fuse_tcp_pairs() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (cached[dev] > 0) return cached[dev];
+  const size_t smem = sizeof(pf::Smem) + 1024;
+  if (cudaFuncSetAttribute(pf::fuse_v_tcp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess)
+    return 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2, 1, 1);
+  cfg.blockDim = dim3(pf::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, pf::fuse_v_tcp_kernel, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    int sms = 2;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    n = std::max(1, sms / 2);
+  }
+  cached[dev] = n;
+  return n;
+}
 
 cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const Tables& tb,
                            const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
@@ -505,18 +616,29 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  CUtensorMap m128, m64, m32;
-  if (!make_rows_map(&m128, Vs, (uint64_t)vs_rows, kTile) || !make_rows_map(&m64, Vs, (uint64_t)vs_rows, 64) ||
-      !make_rows_map(&m32, Vs, (uint64_t)vs_rows, 32))
+  if (units == 0) return cudaSuccess;
+  CUtensorMap m128, m64;
+  if (!make_rows_map(&m128, Vs, (uint64_t)vs_rows, pf::kTile) ||
+      !make_rows_map(&m64, Vs, (uint64_t)vs_rows, pf::kDHalf))
     return cudaErrorInvalidValue;
-  const size_t smem = sizeof(FSmem) + 1024;
-  cudaError_t e = cudaFuncSetAttribute(fuse_v_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const size_t smem = sizeof(pf::Smem) + 1024;
+  cudaError_t e = cudaFuncSetAttribute(pf::fuse_v_tcp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
+  const int pairs = std::max(1, fuse_tcp_pairs());
   ProfileScope ps("fuse_v_tc", st);
-  fuse_v_tc_kernel<<<2 * units, kThreads, smem, st>>>(m128, m64, m32, sh, tb, mu, kLog2e / tau,
-                                                      static_cast<__nv_bfloat16*>(V_out));
-  return cudaGetLastError();
+  // one launch per slice of at most pairs * kMaxUnits units (one for every
+  // workload here), each pair holding at most kMaxUnits descriptors
+  const int64_t per_launch = (int64_t)pairs * pf::kMaxUnits;
+  for (int64_t o = 0; o < units; o += per_launch) {
+    const int cnt = (int)std::min<int64_t>(per_launch, units - o);
+    const int p = std::min(pairs, cnt);
+    pf::fuse_v_tcp_kernel<<<2 * p, pf::kThreads, smem, st>>>(m128, m64, sh, tb, units, (int)o, cnt, mu,
+                                                             kLog2e / tau, static_cast<__nv_bfloat16*>(V_out));
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace vc

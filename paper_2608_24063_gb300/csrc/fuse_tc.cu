@@ -207,12 +207,16 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
   const uint32_t rank = cluster_rank();
   const int pair = (int)(blockIdx.x >> 1), npairs = (int)(gridDim.x >> 1);
   // this launch covers positions [o_lo, o_lo + o_cnt) of the longest-first unit
-  // order (position o is unit units-1-o); pair p takes o_lo + p, o_lo + p + P, ...
-  const int nunits = min(kMaxUnits, (o_cnt - pair + npairs - 1) / npairs);
+  // order (position o is unit units-1-o), dealt to the pairs back and forth:
+  // in round i pair p takes position i*P + p (i even) or i*P + P-1-p (i odd),
+  // so every pair gets long and short units alike
+  const int rounds = o_cnt / npairs, rem = o_cnt % npairs;
+  const int nunits = min(kMaxUnits, rounds + ((rounds & 1) ? (pair >= npairs - rem) : (pair < rem)));
 
   // this pair's unit descriptors
   for (int i = threadIdx.x; i < nunits; i += kThreads) {
-    const int unit = units - 1 - (o_lo + pair + i * npairs);
+    const int pos = i * npairs + ((i & 1) ? npairs - 1 - pair : pair);
+    const int unit = units - 1 - (o_lo + pos);
     const int rl = upper_index(tb.unit0_fuse_tc, sh.n_req * sh.L, (int32_t)unit);
     const Req rq = tb.req[rl / sh.L];
     const Layer ly = tb.layer[rl];

@@ -10,10 +10,12 @@
 // problem; many CTAs per problem, ranks exact and schedule-independent.
 //
 // compact_kernel: one CTA per (request, layer <= h, KV head) with B_l > 0.  A
-// block-wide scan over tokens in ascending position emits keep = {rank < B_l}
-// and drop = {B_l <= rank < Nq}, so both lists come out ascending and the
-// result does not depend on thread scheduling.
+// block-wide scan over tokens in ascending position (segments of 8192
+// consecutive tokens, 8 per thread) emits keep = {rank < B_l} and drop =
+// {B_l <= rank < Nq}, so both lists come out ascending and the result does
+// not depend on thread scheduling.
 #include <algorithm>
+#include <climits>
 
 #include "vc_common.cuh"
 #include "kernels.h"
@@ -139,12 +141,14 @@ __global__ void __launch_bounds__(kSortChunk) chunk_rank_kernel(Shape sh, Tables
 
 // One CTA per (request, layer, KV head); layers with B_l == 0 exit at once.
 constexpr int kScanThreads = 1024;
+constexpr int kScanPer = 8;                  // tokens per thread per segment
 
 __global__ void __launch_bounds__(kScanThreads) compact_kernel(Shape sh, Tables tb,
                                                                const int32_t* __restrict__ rank,
                                                                int32_t* __restrict__ keep_idx,
                                                                int32_t* __restrict__ drop_idx) {
-  __shared__ int32_t wk[32], wd[32];
+  constexpr int kWarps = kScanThreads / 32;
+  __shared__ int32_t wk[kWarps], wd[kWarps], tot[2];
   const int g = blockIdx.y;
   const int rl = blockIdx.x;                 // request * L + layer
   const int r = rl / sh.L, l = rl % sh.L;
@@ -157,49 +161,61 @@ __global__ void __launch_bounds__(kScanThreads) compact_kernel(Shape sh, Tables 
                                              : (int64_t)g * n);
   int32_t* ko = keep_idx + rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B;
   int32_t* dro = drop_idx + rq.drop_row0 + (int64_t)sh.Hkv * ly.Qd + (int64_t)g * ly.D;
-  const int per = (n + kScanThreads - 1) / kScanThreads;
-  const int t0 = threadIdx.x * per;
-  const int t1 = min(n, t0 + per);
-  int ck = 0, cd = 0;
-  for (int v = t0; v < t1; ++v) {
-    const int x = rk[v];
-    ck += x < ly.B;
-    cd += (x >= ly.B) & (x < rq.Nq);
-  }
-  // block exclusive scan of (ck, cd)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int ik = ck, id = cd;
+  // segments of kScanThreads * kScanPer consecutive tokens: thread t looks at
+  // tokens s + t*kScanPer ..., the block counts the keep/drop tokens before
+  // them (warp scans, warp totals through shared memory) and the thread
+  // writes its own at the running offsets, so both lists come out in
+  // ascending position
+  int base_k = 0, base_d = 0;
+  for (int s0 = 0; s0 < n; s0 += kScanThreads * kScanPer) {
+    const int v0 = s0 + (int)threadIdx.x * kScanPer;
+    int xs[kScanPer];
 #pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int a = __shfl_up_sync(0xffffffffu, ik, off);
-    const int b = __shfl_up_sync(0xffffffffu, id, off);
-    if (lane >= off) { ik += a; id += b; }
-  }
-  if (lane == 31) { wk[warp] = ik; wd[warp] = id; }
-  __syncthreads();
-  if (warp == 0) {
-    int a = wk[lane], b = wd[lane];
-    int ia = a, ib = b;
+    for (int k = 0; k < kScanPer; ++k) xs[k] = v0 + k < n ? rk[v0 + k] : INT_MAX;
+    int ck = 0, cd = 0;
+#pragma unroll
+    for (int k = 0; k < kScanPer; ++k) {
+      ck += xs[k] < ly.B;
+      cd += (xs[k] >= ly.B) & (xs[k] < rq.Nq);
+    }
+    int ik = ck, id = cd;                    // inclusive warp scan
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
-      const int x = __shfl_up_sync(0xffffffffu, ia, off);
-      const int y = __shfl_up_sync(0xffffffffu, ib, off);
-      if (lane >= off) { ia += x; ib += y; }
+      const int a = __shfl_up_sync(0xffffffffu, ik, off);
+      const int b = __shfl_up_sync(0xffffffffu, id, off);
+      if (lane >= off) { ik += a; id += b; }
     }
-    wk[lane] = ia - a;
-    wd[lane] = ib - b;
-  }
-  __syncthreads();
-  int pk = wk[warp] + ik - ck, pd = wd[warp] + id - cd;
-  for (int v = t0; v < t1; ++v) {
-    const int x = rk[v];
-    if (x < ly.B) {
-      if (pk < ly.B) ko[pk] = v; else set_status(tb.status, VC_ERR_DEVICE_INDEX);
-      ++pk;
-    } else if (x < rq.Nq) {
-      if (pd < ly.D) dro[pd] = v; else set_status(tb.status, VC_ERR_DEVICE_INDEX);
-      ++pd;
+    if (lane == 31) { wk[warp] = ik; wd[warp] = id; }
+    __syncthreads();
+    if (warp == 0) {                         // exclusive scan of the warp totals, and the block total
+      const int a = lane < kWarps ? wk[lane] : 0, b = lane < kWarps ? wd[lane] : 0;
+      int ia = a, ib = b;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, ia, off);
+        const int y = __shfl_up_sync(0xffffffffu, ib, off);
+        if (lane >= off) { ia += x; ib += y; }
+      }
+      if (lane < kWarps) { wk[lane] = ia - a; wd[lane] = ib - b; }
+      if (lane == 31) { tot[0] = ia; tot[1] = ib; }
     }
+    __syncthreads();
+    int pk = base_k + wk[warp] + ik - ck, pd = base_d + wd[warp] + id - cd;
+#pragma unroll
+    for (int k = 0; k < kScanPer; ++k) {
+      const int x = xs[k], v = v0 + k;
+      if (x < ly.B) {
+        if (pk < ly.B) ko[pk] = v; else set_status(tb.status, VC_ERR_DEVICE_INDEX);
+        ++pk;
+      } else if (x < rq.Nq) {
+        if (pd < ly.D) dro[pd] = v; else set_status(tb.status, VC_ERR_DEVICE_INDEX);
+        ++pd;
+      }
+    }
+    base_k += tot[0];
+    base_d += tot[1];
+    __syncthreads();                         // shared totals are rewritten next segment
   }
 }
 

@@ -90,20 +90,8 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
 // ---------------------------------------------------------------------------
 // shared helpers of the fusion
 
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  const uint32_t a = smem_u32(p);
-  return p + ((1024u - (a & 1023u)) & 1023u);
-}
 
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
-  int dummy = 0;
-  mbar_wait(bar, parity, &dummy);
-}
 
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const bool ok = mbar_wait(bar, parity, abort);
-  return __all_sync(0xffffffffu, ok);
-}
 
 // Byte offset of 16-byte chunk c (0..7) of row r in a 128-byte-swizzled
 // K-block (the layout TMA writes and the MMA descriptors expect).
@@ -193,6 +181,8 @@ struct Smem {
   uint64_t lsum_empty[2];              // own: the 4 epilogue warps read them
   uint64_t mma_done;                   // both: every MMA of the pair is done
   uint64_t never;                      // test support: never completes
+  uint64_t peer_done;                  // even CTA: the odd CTA's fill count landed (8 bytes)
+  int2 peer_fills;                     // even CTA: dropped tiles the odd CTA issued
   uint32_t tmem_base;
   int abort;
 };
@@ -249,8 +239,10 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
     for (int i = 0; i < kStages; ++i) { mbar_init(&sm.vd_full[i], 1); mbar_init(&sm.vd_empty[i], 1); }
     mbar_init(&sm.mma_done, 1);
     mbar_init(&sm.never, 1);
+    mbar_init(&sm.peer_done, 1);
     sm.abort = 0;
     fence_mbar_init();
+    if (rank == 0) mbar_arrive_expect_tx(&sm.peer_done, 8);
   }
   if (warp == kProducerWarp) {
     tmem_alloc_pair(&sm.tmem_base, kTmemCols);
@@ -289,10 +281,15 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
         ++t;
       }
     }
-    // every copy this CTA started has landed before the pair may leave
+    // every copy this CTA started has landed before the pair may leave: the
+    // kept rows on this CTA's barriers, the dropped tiles (both halves) on the
+    // even CTA's, drained there with the odd CTA's count of them
+    if (rank == 1) report_fills(&sm.peer_fills, &sm.peer_done, t, 0);
     for (int i = max(0, kl - 2); i < kl; ++i) drain_wait(&sm.vk_full[i & 1], (i >> 1) & 1);
-    if (rank == 0)
-      for (int i = max(0, t - kStages); i < t; ++i) drain_wait(&sm.vd_full[i % kStages], (i / kStages) & 1);
+    if (rank == 0) {
+      const int2 f = peer_fills(&sm.peer_done, &sm.peer_fills, make_int2(t, 0), abort);
+      drain_pair_ring(sm.vd_full, kStages, t, f.x, 2 * kDHalfKB + kDKB);
+    }
   } else if (warp == kProducerWarp && lane == 1) {
     // ---- kept-rows relay: this CTA's kept rows of unit k landed -> even CTA
     const uint32_t pair0 = map_to_rank(smem_u32(&sm.vk_pair[0]), 0);
@@ -355,17 +352,26 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
     // always committed (also after a give-up), so every wait on it ends
     mma_commit_pair(&sm.mma_done, 3);
     drain_wait(&sm.mma_done, 0);
+  } else if (warp == kMmaWarp && lane == 0) {
+    // odd CTA: the pair's MMAs (and their arrivals on this CTA's barriers) are done
+    drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
     if ((sh.test_wait & VC_TEST_WAIT_FUSE) && warp == 0) {
-      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) {
+        set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+        *abort = 1;
+      }
       __syncwarp();
     }
     // ---- softmax over the drop set: one kept row per TMEM lane
     const int q4 = warp & 3, hf = warp >> 2;
     const uint32_t lane_off = (uint32_t)(q4 << 5) << 16;
+    // After a give-up the warp stays in its loops without waiting, touching
+    // tensor memory or arriving, but still meets its partner warp at every
+    // named barrier (the partner may not have given up).
     int t = 0;
     bool ok = true;
-    for (int k = 0; ok && k < nunits; ++k) {
+    for (int k = 0; k < nunits; ++k) {
       const Unit d = sm.unit[k];
       const int b = k & 1;
       const int nt = (d.D + (int)kDTile - 1) / (int)kDTile;
@@ -373,7 +379,11 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
       float m = -INFINITY, lsum = 0.f;
       for (int j = 0; j < nt; ++j, ++t) {
         const int bsel = t & 1;
-        if (!warp_wait(&sm.s_full[bsel], (t >> 1) & 1, abort)) { ok = false; break; }
+        ok = ok && warp_wait(&sm.s_full[bsel], (t >> 1) & 1, abort);
+        if (!ok) {
+          named_sync(1 + q4, 64);
+          continue;
+        }
         tc_fence_after();
         const uint32_t s_col = tbase + lane_off + kSCol + (uint32_t)bsel * kDTile + (uint32_t)hf * 64;
         float x[4][16];
@@ -434,26 +444,29 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
           // rare: rescale this warp's 64 columns of O[b] once O(t-1) is done (its
           // commit frees stage (t-1) % kStages); O(t) waits for P(t), below
           const int tp = t - 1;
-          if (!warp_wait(&sm.vd_empty[tp % kStages], (tp / kStages) & 1, abort)) { ok = false; break; }
-          tc_fence_after();
+          ok = warp_wait(&sm.vd_empty[tp % kStages], (tp / kStages) & 1, abort);
+          if (ok) {
+            tc_fence_after();
 #pragma unroll 1
-          for (int p = 0; p < 4; ++p) {
-            uint32_t v[16];
-            tmem_ld16(o_col + p * 16, v);
-            tmem_wait(v);
+            for (int p = 0; p < 4; ++p) {
+              uint32_t v[16];
+              tmem_ld16(o_col + p * 16, v);
+              tmem_wait(v);
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
-            tmem_st16(o_col + p * 16, v);
+              for (int q = 0; q < 16; ++q) v[q] = __float_as_uint(__uint_as_float(v[q]) * corr);
+              tmem_st16(o_col + p * 16, v);
+            }
           }
         }
         tmem_wait_st();
+        if (!ok) continue;
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(map_to_rank(smem_u32(&sm.p_full[bsel]), 0));
       }
-      if (!ok) break;
       // the unit's row sums, once the epilogue has read those of unit k - 2
-      if (!warp_wait(&sm.lsum_empty[b], ((k >> 1) & 1) ^ 1, abort)) break;
+      ok = ok && warp_wait(&sm.lsum_empty[b], ((k >> 1) & 1) ^ 1, abort);
+      if (!ok) continue;
       sm.lsum[b][q4][hf][lane] = lsum;
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.lsum_full[b]);
@@ -466,74 +479,80 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
     const uint32_t o_empty0 = map_to_rank(smem_u32(&sm.o_empty[0]), 0);
     const uint32_t o_empty1 = map_to_rank(smem_u32(&sm.o_empty[1]), 0);
     const int te = (warp - kEpiWarp0) * 32 + lane;    // 0..127
+    // After a give-up the warp keeps meeting the other epilogue warps at both
+    // named barriers of every unit, and no warp copies a unit out once any of
+    // them has given up.
+    bool ok = true;
     for (int k = 0; k < nunits; ++k) {
       const Unit d = sm.unit[k];
       const int b = k & 1;
       const uint32_t ph = (k >> 1) & 1;
-      if (!warp_wait(&sm.vk_full[b], ph, abort) || !warp_wait(&sm.lsum_full[b], ph, abort) ||
-          !warp_wait(&sm.o_full[b], ph, abort))
-        break;
-      tc_fence_after();
-      const bool have_o = d.D > 0;
-      const float lt = sm.lsum[b][q4][0][lane] + sm.lsum[b][q4][1][lane];   // same order as fuse_v_tc
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.lsum_empty[b]);
-      const float w_o = have_o ? (1.f - mu) / lt : 0.f;
-      const float w_k = have_o ? mu : 1.f;
-      const uint32_t o_col = tbase + lane_off + (uint32_t)b * kTile;
+      ok = ok && warp_wait(&sm.vk_full[b], ph, abort) && warp_wait(&sm.lsum_full[b], ph, abort) &&
+           warp_wait(&sm.o_full[b], ph, abort);
+      if (ok) {
+        tc_fence_after();
+        const bool have_o = d.D > 0;
+        const float lt = sm.lsum[b][q4][0][lane] + sm.lsum[b][q4][1][lane];   // same order as fuse_v_tc
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.lsum_empty[b]);
+        const float w_o = have_o ? (1.f - mu) / lt : 0.f;
+        const float w_k = have_o ? mu : 1.f;
+        const uint32_t o_col = tbase + lane_off + (uint32_t)b * kTile;
 #pragma unroll 1
-      for (int hh = 0; hh < 4; ++hh) {                // 32 output columns at a time
-        float o[2][16];
-        if (have_o) {
-          uint32_t v[2][16];
+        for (int hh = 0; hh < 4; ++hh) {                // 32 output columns at a time
+          float o[2][16];
+          if (have_o) {
+            uint32_t v[2][16];
 #pragma unroll
-          for (int p = 0; p < 2; ++p) tmem_ld16(o_col + hh * 32 + p * 16, v[p]);
-          tmem_wait_only();
+            for (int p = 0; p < 2; ++p) tmem_ld16(o_col + hh * 32 + p * 16, v[p]);
+            tmem_wait_only();
 #pragma unroll
-          for (int p = 0; p < 2; ++p) {
-            reg_fence(v[p]);
+            for (int p = 0; p < 2; ++p) {
+              reg_fence(v[p]);
 #pragma unroll
-            for (int q = 0; q < 16; ++q) o[p][q] = __uint_as_float(v[p][q]);
+              for (int q = 0; q < 16; ++q) o[p][q] = __uint_as_float(v[p][q]);
+            }
+          } else {
+#pragma unroll
+            for (int p = 0; p < 2; ++p)
+#pragma unroll
+              for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
           }
-        } else {
+          const int kb = hh >> 1;
 #pragma unroll
-          for (int p = 0; p < 2; ++p)
+          for (int c4 = 0; c4 < 4; ++c4) {
+            const int c8 = (hh & 1) * 4 + c4;             // 16-byte chunk within K-block kb
+            const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[b][kb][0] + swz(row, c8));
+            const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
+            uint4 w;
+            uint32_t* wp = &w.x;
 #pragma unroll
-            for (int q = 0; q < 16; ++q) o[p][q] = 0.f;
+            for (int q = 0; q < 4; ++q) {
+              const float2 kf = __bfloat1622float2(k2[q]);
+              const float a = fmaf(w_k, kf.x, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q]);
+              const float bb = fmaf(w_k, kf.y, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q + 1]);
+              wp[q] = pack_bf16x2(a, bb);
+            }
+            const int c = kb * 8 + c8;
+            *reinterpret_cast<uint4*>(&sm.stg[0] + row * 256 + ((c ^ (row & 15)) << 4)) = w;
+          }
         }
-        const int kb = hh >> 1;
-#pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
-          const int c8 = (hh & 1) * 4 + c4;             // 16-byte chunk within K-block kb
-          const uint4 kv = *reinterpret_cast<const uint4*>(&sm.vk[b][kb][0] + swz(row, c8));
-          const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&kv);
-          uint4 w;
-          uint32_t* wp = &w.x;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float2 kf = __bfloat1622float2(k2[q]);
-            const float a = fmaf(w_k, kf.x, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q]);
-            const float bb = fmaf(w_k, kf.y, w_o * o[c4 >> 1][(c4 & 1) * 8 + 2 * q + 1]);
-            wp[q] = pack_bf16x2(a, bb);
-          }
-          const int c = kb * 8 + c8;
-          *reinterpret_cast<uint4*>(&sm.stg[0] + row * 256 + ((c ^ (row & 15)) << 4)) = w;
+        // O[b] and vk[b] are read: free them
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive_cluster(b ? o_empty1 : o_empty0);
+          mbar_arrive(&sm.vk_empty[b]);
         }
       }
-      // O[b] and vk[b] are read: free them
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive_cluster(b ? o_empty1 : o_empty0);
-        mbar_arrive(&sm.vk_empty[b]);
-      }
-      named_sync(5, 32 * kEpiWarps);                 // staging complete
+      if (!named_sync_any(5, 32 * kEpiWarps, !ok)) {   // staging complete
 #pragma unroll 4
-      for (int i = 0; i < 16; ++i) {                  // coalesced copy-out, 16 threads per row
-        const int rr = i * 8 + (te >> 4), c = te & 15;
-        if (rr < d.rows)
-          *reinterpret_cast<uint4*>(V_out + (d.orow + rr) * 128 + c * 8) =
-              *reinterpret_cast<const uint4*>(&sm.stg[0] + rr * 256 + ((c ^ (rr & 15)) << 4));
+        for (int i = 0; i < 16; ++i) {                // coalesced copy-out, 16 threads per row
+          const int rr = i * 8 + (te >> 4), c = te & 15;
+          if (rr < d.rows)
+            *reinterpret_cast<uint4*>(V_out + (d.orow + rr) * 128 + c * 8) =
+                *reinterpret_cast<const uint4*>(&sm.stg[0] + rr * 256 + ((c ^ (rr & 15)) << 4));
+        }
       }
       named_sync(5, 32 * kEpiWarps);                 // staging free for the next unit
     }

@@ -54,23 +54,8 @@ constexpr uint32_t kKBlockBytes = kTile * 128;  // 128 rows x 64 bf16
 constexpr uint32_t kTileBytes = 2 * kKBlockBytes;
 constexpr uint32_t kTmemCols = 512;
 
-__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
-  const uint32_t a = smem_u32(p);
-  return p + ((1024u - (a & 1023u)) & 1023u);
-}
 
-// Wait bounded by time only (used when draining after an abort).
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
-  int dummy = 0;
-  mbar_wait(bar, parity, &dummy);
-}
 
-// mbarrier wait whose outcome is the same for all 32 lanes (tcgen05.ld is a
-// warp-wide instruction, so a warp must never split on a wait).
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const bool ok = mbar_wait(bar, parity, abort);
-  return __all_sync(0xffffffffu, ok);
-}
 
 // sum_j exp2(x_j * s + b_j) over 16 values, with packed fp32x2 FMA and adds
 // (pairwise, so the rounding error stays a few ulp).
@@ -113,8 +98,10 @@ struct P1Smem {
   uint64_t k_empty[kStagesPair];            // both: the MMAs reading the stage are done
   uint64_t tm_full[2];                      // both: the slot's logits are ready
   uint64_t tm_empty[2];                     // even CTA: the slot's 8 consumer warps copied it out
-  uint64_t mma_done;
+  uint64_t mma_done;                        // both: every MMA of the pair is done
   uint64_t never;                           // test support: never completes
+  uint64_t peer_done;                       // even CTA: the odd CTA's fill count landed (8 bytes)
+  int2 peer_fills;                          // even CTA: key tiles the odd CTA issued
   uint32_t tmem_base;
   int abort;
 };
@@ -151,8 +138,10 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     for (int i = 0; i < 2; ++i) { mbar_init(&sm.tm_full[i], 1); mbar_init(&sm.tm_empty[i], 8); }
     mbar_init(&sm.mma_done, 1);
     mbar_init(&sm.never, 1);
+    mbar_init(&sm.peer_done, 1);
     sm.abort = 0;
     fence_mbar_init();
+    if (rank == 0) mbar_arrive_expect_tx(&sm.peer_done, 8);
   }
   if (warp == kProducerWarp) {
     tmem_alloc_pair(&sm.tmem_base, kTmemCols);
@@ -183,11 +172,13 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       tma_load_2d_pair(sm.k[st][1], &tmK, 64, y, k_full0);
       ++issued;
     }
-    // the even CTA waits until every copy of both CTAs has landed
+    // the even CTA waits until every copy of both CTAs has landed (both
+    // always issue their Q rows; the key ring with the odd CTA's count)
+    if (rank == 1) report_fills(&sm.peer_fills, &sm.peer_done, issued, 0);
     if (rank == 0) {
       drain_wait(&sm.q_full, 0);
-      for (int i = max(0, issued - kStagesPair); i < issued; ++i)
-        drain_wait(&sm.k_full[i % kStagesPair], (i / kStagesPair) & 1);
+      const int2 f = peer_fills(&sm.peer_done, &sm.peer_fills, make_int2(issued, 0), abort);
+      drain_pair_ring(sm.k_full, kStagesPair, issued, f.x, kTileBytes);
     }
   } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
     // ---- MMA issuer (even CTA): D[row][key] for 256 rows x 256 keys per tile
@@ -209,11 +200,17 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       mma_commit_pair(&sm.tm_full[slot], 3);
       mma_commit_pair(&sm.k_empty[st], 3);
     }
-    mma_commit_pair(&sm.mma_done, 1);
+    mma_commit_pair(&sm.mma_done, 3);
+    drain_wait(&sm.mma_done, 0);
+  } else if (warp == kMmaWarp && lane == 0) {
+    // odd CTA: the pair's MMAs (and their arrivals on this CTA's barriers) are done
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
     if ((sh.test_wait & VC_TEST_WAIT_SCORE_LSE) && warp == 0) {
-      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) {
+        set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+        *abort = 1;
+      }
       __syncwarp();
     }
     // ---- row statistics: one thread per row (= TMEM lane).  Warpgroup wg
@@ -436,8 +433,10 @@ struct P2Smem {
   uint64_t q_empty[kQStagesPair];             // both: MMAs done and this CTA's warpgroup read the normalisers
   uint64_t tm_full[2];                        // both: the slot's logits are ready
   uint64_t tm_empty[2];                       // even CTA: the slot's 8 consumer warps copied it out
-  uint64_t mma_done;
+  uint64_t mma_done;                          // both: every MMA of the pair is done
   uint64_t never;                             // test support: never completes
+  uint64_t peer_done;                         // even CTA: the odd CTA's fill counts landed (8 bytes)
+  int2 peer_fills;                            // even CTA: (key, chunk) tiles the odd CTA issued
   uint32_t tmem_base;
   int abort;
 };
@@ -474,8 +473,10 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     }
     mbar_init(&sm.mma_done, 1);
     mbar_init(&sm.never, 1);
+    mbar_init(&sm.peer_done, 1);
     sm.abort = 0;
     fence_mbar_init();
+    if (rank == 0) mbar_arrive_expect_tx(&sm.peer_done, 8);
   }
   if (warp == kProducerWarp) {
     tmem_alloc_pair(&sm.tmem_base, kTmemCols);
@@ -520,12 +521,13 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     }
     // every copy this CTA started has landed before the pair may leave: the
     // normalisers on this CTA's barriers, the tiles on the even CTA's
+    if (rank == 1) report_fills(&sm.peer_fills, &sm.peer_done, k_issued, q_issued);
     for (int i = max(0, q_issued - kQStagesPair); i < q_issued; ++i)
       drain_wait(&sm.nl_full[i % kQStagesPair], (i / kQStagesPair) & 1);
     if (rank == 0) {
-      for (int i = max(0, k_issued - 2); i < k_issued; ++i) drain_wait(&sm.k_full[i & 1], (i >> 1) & 1);
-      for (int i = max(0, q_issued - kQStagesPair); i < q_issued; ++i)
-        drain_wait(&sm.q_full[i % kQStagesPair], (i / kQStagesPair) & 1);
+      const int2 f = peer_fills(&sm.peer_done, &sm.peer_fills, make_int2(k_issued, q_issued), abort);
+      drain_pair_ring(sm.k_full, 2, k_issued, f.x, kTileBytes);
+      drain_pair_ring(sm.q_full, kQStagesPair, q_issued, f.y, kTileBytes);
     }
   } else if (warp == kMmaWarp && lane == 0 && rank == 0) {
     // ---- MMA issuer (even CTA): D[key][row] = K_tile . Q_chunk^T, 256 x cw
@@ -551,11 +553,17 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
       }
       if (ok) mma_commit_pair(&sm.k_empty[ks], 3);
     }
-    mma_commit_pair(&sm.mma_done, 1);
+    mma_commit_pair(&sm.mma_done, 3);
+    drain_wait(&sm.mma_done, 0);
+  } else if (warp == kMmaWarp && lane == 0) {
+    // odd CTA: the pair's MMAs (and their arrivals on this CTA's barriers) are done
     drain_wait(&sm.mma_done, 0);
   } else if (warp < 8) {
     if ((sh.test_wait & VC_TEST_WAIT_SCORE_COLSUM) && warp == 0) {
-      if (lane == 0 && injected_wait_gives_up(&sm.never)) set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+      if (lane == 0 && injected_wait_gives_up(&sm.never)) {
+        set_status(tb.status, VC_ERR_DEVICE_TIMEOUT);
+        *abort = 1;
+      }
       __syncwarp();
     }
     // ---- column sums: one thread per key (= TMEM lane)

@@ -22,6 +22,11 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  const uint32_t a = smem_u32(p);
+  return p + ((1024u - (a & 1023u)) & 1023u);
+}
+
 // ---------------------------------------------------------------------------
 // mbarriers
 
@@ -90,6 +95,26 @@ constexpr long long kTestWaitCycles = 100000;
 
 __device__ __forceinline__ bool injected_wait_gives_up(uint64_t* never) {
   return !mbar_wait_for(never, 0, kTestWaitCycles);
+}
+
+// Wait bounded by time only (used when draining after an abort).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  int dummy = 0;
+  mbar_wait(bar, parity, &dummy);
+}
+
+// mbarrier wait whose outcome is the same for all 32 lanes (tcgen05.ld is a
+// warp-wide instruction, so a warp must never split on a wait).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, abort);
+  return __all_sync(0xffffffffu, ok);
+}
+
+// complete-tx of `bytes` on an mbarrier of this CTA with no copy behind it:
+// stands in for bytes that will never be sent (drain_pair_ring).
+__device__ __forceinline__ void mbar_complete_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -329,6 +354,68 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t ran
 // it.  A cluster-scope release here costs about a thousand cycles.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Pair-counted rings.  A stage of such a ring is filled by both CTAs: each
+// copies its own half into its own shared memory, and both copies count
+// their bytes on the even CTA's barrier, which the even CTA arms for the two
+// halves.  After an abort the two loaders may stop at different fills, so
+// neither side alone knows which copies are still in flight.  The odd CTA
+// reports its fill counts (report_fills) and the even CTA drains the ring
+// with them (drain_pair_ring) before the pair may leave.
+
+// The odd CTA tells the even CTA how many fills of up to two pair-counted
+// rings it issued: an 8-byte store into the even CTA's `dst` whose bytes
+// complete on the even CTA's barrier `done` (armed there for 8 bytes).
+__device__ __forceinline__ void report_fills(int2* dst, uint64_t* done, int n_a, int n_b) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.s32 [%0], {%2, %3}, [%1];" ::"r"(
+                   map_to_rank(smem_u32(dst), 0)),
+               "r"(map_to_rank(smem_u32(done), 0)), "r"(n_a), "r"(n_b)
+               : "memory");
+}
+
+// Even CTA, after both loaders stopped: wait until every copy counted on the
+// ring `full` of `stages` barriers has landed.  The even CTA armed fills
+// 0 .. n0-1 (and issued its halves), the odd CTA issued its halves of fills
+// 0 .. n1-1.  Either CTA issues fill i only after the stage's consumer
+// released fill i - stages, which it did only after fill i - stages
+// completed; so |n0 - n1| <= stages and every fill below n0 - stages has
+// completed.  A fill of the window that the odd CTA never issued gets its
+// half's bytes by a bare complete-tx; one that only the odd CTA issued is
+// armed for its half alone.  Each wait is bounded.
+__device__ __forceinline__ void drain_pair_ring(uint64_t* full, int stages, int n0, int n1,
+                                                uint32_t peer_bytes) {
+  n1 = max(n0 - stages, min(n0 + stages, n1));
+  for (int i = max(0, n0 - stages); i < max(n0, n1); ++i) {
+    uint64_t* b = &full[i % stages];
+    if (i >= n0) mbar_arrive_expect_tx(b, peer_bytes);
+    else if (i >= n1) mbar_complete_tx(b, peer_bytes);
+    drain_wait(b, (uint32_t)(i / stages) & 1u);
+  }
+}
+
+// The odd CTA's fill counts once its report has landed (bounded wait: the
+// odd loader reports within about one wait limit of stopping); `fallback`
+// when it never comes, in which case *abort is set.
+__device__ __forceinline__ int2 peer_fills(uint64_t* done, const int2* fills, int2 fallback,
+                                           volatile int* abort) {
+  if (mbar_wait_for(done, 0, 3 * kWaitCycles)) return *fills;
+  *abort = 1;
+  return fallback;
+}
+
+// Named barrier that also reports whether `pred` held in any of the threads.
+__device__ __forceinline__ bool named_sync_any(uint32_t id, uint32_t threads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.or.pred p, %2, %3, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(threads)
+      : "memory");
+  return r != 0;
 }
 
 // 2-D tile load into this CTA's shared memory whose completion is counted on

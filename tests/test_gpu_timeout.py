@@ -2,17 +2,23 @@
 
 Every wait of the tensor-core kernels (score_lse_tc, score_colsum_tc, fuse_v_tc)
 is bounded and records VC_ERR_DEVICE_TIMEOUT in the workspace status word when
-it gives up.  viscache_test_inject_wait makes one consumer warp of the chosen
-kernel wait on an mbarrier that nothing ever completes (a flag that nothing
-sets), with a short limit; the wait must give up, the host must read the
-timeout through prunekv_get_status (or prunekv_score_static_status for the
-fixed-scratch entry point), and the context must stay usable: the same calls
-without the injected wait then return VC_OK and match the fp64 oracle.  The
-injected wait touches none of the kernel's own barriers or copies, so the
-timed-out launch still completes its work (its outputs equal the clean
-launch's bit for bit).
+it gives up.  viscache_test_inject_wait makes one consumer warp of every CTA of
+the chosen kernel wait on an mbarrier that nothing ever completes (a flag that
+nothing sets), with a short limit; when that wait gives up the warp records the
+timeout and raises the CTA's abort flag, exactly as a real give-up does.  The
+rest of the CTA pair then takes the abort path: waits stop, the MMA issuer
+stops issuing, warps that gave up keep meeting their named barriers without
+working, the even CTA drains the pair's copies with the odd CTA's fill counts,
+both CTAs wait for the pair's last MMA, and only then is tensor memory freed.
+
+The checks: the launch returns (well inside the device wait limits), the host
+reads the timeout through prunekv_get_status (or prunekv_score_static_status
+for the fixed-scratch entry point), and the context stays usable: the same
+calls without the injected wait return VC_OK and match the fp64 oracle.  The
+aborted launch's outputs are incomplete by design and are not compared.
 """
 import ctypes
+import time
 
 import numpy as np
 import pytest
@@ -26,6 +32,10 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 L, Hq, Hkv, d, n, W = 3, 14, 2, 128, 2049, 20
 RR = (23, 100)
+# An aborted launch ends within a few device wait limits (each about a second)
+# even when one CTA of a pair gives up long before the other; with every CTA
+# aborting at once it ends in milliseconds.
+ABORT_SECONDS = 30.0
 
 
 def _inputs():
@@ -59,8 +69,10 @@ def test_wait_gives_up_reports_timeout_and_context_stays_usable(mask, where, inj
     Q, K, V = q.to(DEV), k.to(DEV), v.to(DEV)
     B, Nq, _ = vc.viscache_plan_budgets(L, n, *RR)
     inject(mask)
-    bad, st_s, st_f = _steps(Q, K, V, B, Nq)
+    t0 = time.perf_counter()
+    _, st_s, st_f = _steps(Q, K, V, B, Nq)
     torch.cuda.synchronize()
+    assert time.perf_counter() - t0 < ABORT_SECONDS
     assert (st_s, st_f) == ((vc.VC_ERR_DEVICE_TIMEOUT, vc.VC_OK) if where == "score"
                             else (vc.VC_OK, vc.VC_ERR_DEVICE_TIMEOUT))
     inject(0)
@@ -68,8 +80,6 @@ def test_wait_gives_up_reports_timeout_and_context_stays_usable(mask, where, inj
     torch.cuda.synchronize()
     assert (st_s, st_f) == (vc.VC_OK, vc.VC_OK)
     check_request(q, k, v, B, Nq, good, 0.7, 1.0)
-    for key in good:
-        assert torch.equal(bad[key], good[key]), key
 
 
 def test_fused_pass_and_static_scoring_report_timeouts(inject):
@@ -89,15 +99,19 @@ def test_fused_pass_and_static_scoring_report_timeouts(inject):
         return vc.lib().prunekv_score_static_status(stream)
 
     inject(vc.VC_TEST_WAIT_SCORE_LSE | vc.VC_TEST_WAIT_SCORE_COLSUM | vc.VC_TEST_WAIT_FUSE)
-    out_bad = vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
+    t0 = time.perf_counter()
+    vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
     assert vc.prunekv_get_status(ws) == vc.VC_ERR_DEVICE_TIMEOUT
     assert static_call() == vc.VC_ERR_DEVICE_TIMEOUT
+    assert time.perf_counter() - t0 < 2 * ABORT_SECONDS
     inject(0)
     out = vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
     assert vc.prunekv_get_status(ws) == vc.VC_OK
     assert static_call() == vc.VC_OK
     torch.cuda.synchronize()
-    for a, b in zip(out_bad, out):
-        assert torch.equal(a, b)
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, *RR)
+    check_request(q, k, v, B, Nq, _steps(Q, K, V, B, Nq)[0], 0.7, 1.0)
     assert torch.equal(s_static, vc.prunekv_score(Q, K))
+    Ko, Vo, _ = out
+    assert not bool(torch.isnan(Ko.float()).any()) and not bool(torch.isnan(Vo.float()).any())
 

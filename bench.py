@@ -88,8 +88,8 @@ def plans_for(wl, vc, schedule="parabola", drop="survivors"):
 
 def algorithmic(wl, plans):
     eb = 2 if wl.dtype == "bf16" else 4
-    tot = dict(bytes=0, flops_score=0, flops_fuse=0, k_bytes=0, gather_bytes=0, fuse_bytes=0, surv_v_bytes=0,
-               tokens_layers=0)
+    tot = dict(bytes=0, flops_score=0, flops_fuse=0, k_bytes=0, gather_bytes=0, gather_v_bytes=0,
+               gather_kv_bytes=0, fuse_bytes=0, surv_v_bytes=0, tokens_layers=0)
     for r, (B, Nq, h) in zip(wl.requests, plans):
         T = sum(B)
         row = wl.d * eb
@@ -100,7 +100,9 @@ def algorithmic(wl, plans):
         out = 2 * wl.Hkv * T * row
         tot["bytes"] += k_all + q + kept_k + surv_v + out
         tot["k_bytes"] += k_all + q
-        tot["gather_bytes"] += 2 * kept_k
+        tot["gather_bytes"] += 2 * kept_k              # kept keys read and written
+        tot["gather_v_bytes"] += 2 * surv_v            # survivor values read, slab written
+        tot["gather_kv_bytes"] += 2 * (kept_k + surv_v)
         tot["fuse_bytes"] += surv_v + wl.Hkv * T * row
         tot["surv_v_bytes"] += surv_v
         tot["flops_score"] += 2 * wl.Hq * r.W * r.n * wl.d * wl.L
@@ -117,7 +119,8 @@ KERNEL_WORK = {
     "score_colsum_tc": ("tensor", "flops_score"),
     "fuse_v_simt": ("tensor", "flops_fuse"),
     "fuse_v_tc": ("tensor", "flops_fuse"),
-    "gather_kv": ("hbm", "gather_bytes"),
+    "gather_kv": ("hbm", "gather_kv_bytes"),
+    "gather_v": ("hbm", "gather_v_bytes"),
     "gather_k": ("hbm", "gather_bytes"),
 }
 

@@ -304,6 +304,17 @@ cudaError_t launch_score(int dtype, const void* Qw, const void* K, Layout& lay, 
                            scores, st);
 }
 
+// True when p is ordinary device memory (the fusion's key warps read K only
+// then; host or managed memory is left to the gather kernel).
+bool on_device(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice;
+}
+
 // Prune keys and fuse values, Eq. (redistribution, weight_fusion): one tensor-core
 // kernel for bf16, d = 128 (it also copies the kept keys), else the key gather and
 // the CUDA-core fusion.
@@ -312,7 +323,7 @@ cudaError_t launch_fuse(int dtype, const void* K, const void* V, const Layout& l
                         float mu, float tau, void* K_out, void* V_out, uint8_t* w, cudaStream_t st) {
   if (g_path.load() == VC_PATH_AUTO && dtype == VC_BF16 && lay.d == 128 && lay.need_vs)
     return launch_fuse_tc(K, V, sh, tb, keep, drop, mu, tau, K_out, V_out, w + lay.o_vs,
-                          lay.vs_rows, lay.units_gather, lay.units_fuse_tc, st);
+                          lay.vs_rows, on_device(K), lay.units_gather, lay.units_fuse_tc, st);
   cudaError_t e = launch_gather_k(dtype, K, sh, tb, keep, K_out, lay.out_rows, st);
   if (e != cudaSuccess) return e;
   return launch_fuse_simt(dtype, V, sh, tb, keep, drop, mu, tau, V_out, lay.units_fuse, st);

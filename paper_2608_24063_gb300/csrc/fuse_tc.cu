@@ -38,11 +38,12 @@ constexpr int kGatherRows = 16 * kGatherRowsPerThread;   // rows per block
 
 // Each thread copies its 16-byte chunk of four rows (i, i+16, i+32, i+48 of
 // the block), all index loads and then all row loads in flight before the
-// stores, so the dependent loads overlap.
+// stores, so the dependent loads overlap.  keys = 0 leaves K_out to the
+// fusion (it copies the kept keys while its products run).
 __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
     const uint4* __restrict__ K, const uint4* __restrict__ V, Shape sh, Tables tb,
     const int32_t* __restrict__ keep_idx, const int32_t* __restrict__ drop_idx,
-    uint4* __restrict__ K_out, uint4* __restrict__ Vs) {
+    uint4* __restrict__ K_out, uint4* __restrict__ Vs, int keys) {
   const int rl = upper_index(tb.unit0_gather, sh.n_req * sh.L, (int32_t)blockIdx.x);
   const int r = rl / sh.L, l = rl % sh.L;
   const Req rq = tb.req[r];
@@ -74,7 +75,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
     if (v[k] >= 0) {
       const int64_t src = src0 + (int64_t)v[k] * 16;
       vv[k] = V[src];
-      if (i0 + 16 * k < ly.B) kv[k] = K[src];
+      if (keys && i0 + 16 * k < ly.B) kv[k] = K[src];
     }
   }
 #pragma unroll
@@ -82,7 +83,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
     const int i = i0 + 16 * k;
     if (v[k] >= 0) {
       Vs[(sbase + i) * 16 + c] = vv[k];
-      if (i < ly.B) K_out[(kbase + i) * 16 + c] = kv[k];
+      if (keys && i < ly.B) K_out[(kbase + i) * 16 + c] = kv[k];
     }
   }
 }
@@ -138,7 +139,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 namespace pf {
 
 constexpr int kProducerWarp = 8, kMmaWarp = 9, kEpiWarp0 = 10, kEpiWarps = 4;
-constexpr int kThreads = 32 * (kEpiWarp0 + kEpiWarps);   // 448
+constexpr int kKeyWarp0 = kEpiWarp0 + kEpiWarps, kKeyWarps = 2;
+constexpr int kThreads = 32 * (kKeyWarp0 + kKeyWarps);   // 512
 constexpr uint32_t kTile = 128;                  // kept rows per CTA
 constexpr uint32_t kKB = kTile * 128;            // 128 rows x 128 bytes
 constexpr uint32_t kDTile = 128;                 // dropped rows per tile (both CTAs)
@@ -156,8 +158,9 @@ struct Unit {              // one unit as this CTA sees it
   int32_t vd_row;          // Vs row of the (layer, KV head)'s first dropped row
   int32_t D;               // dropped rows
   int32_t rows;            // kept rows of this CTA (0..128)
-  int64_t orow;            // V_out row of this CTA's first kept row
-  int64_t pad;
+  int64_t orow;            // K_out / V_out row (= keep-list position) of this CTA's first kept row
+  int32_t kv_row;          // K row of the (layer, KV head)'s token 0
+  int32_t n;               // tokens of the request
 };
 
 struct Smem {
@@ -190,7 +193,8 @@ struct Smem {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_constant__ CUtensorMap tmRows64,
                   Shape sh, Tables tb, int units, int o_lo, int o_cnt, float mu, float c2,
-                  __nv_bfloat16* __restrict__ V_out) {
+                  __nv_bfloat16* __restrict__ V_out, int kcopy, const int32_t* __restrict__ keep_idx,
+                  const uint4* __restrict__ K, uint4* __restrict__ K_out) {
   extern __shared__ uint8_t smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -221,7 +225,8 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
     d.D = ly.D;
     d.rows = max(0, min((int)kTile, ly.B - r0));
     d.orow = rq.out_row0 + (int64_t)sh.Hkv * ly.P + (int64_t)g * ly.B + r0;
-    d.pad = 0;
+    d.kv_row = (int)(rq.kv_off / 128 + ((int64_t)(rl % sh.L) * sh.Hkv + g) * rq.n);
+    d.n = rq.n;
     sm.unit[i] = d;
   }
   if (threadIdx.x == 0) {
@@ -471,6 +476,54 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.lsum_full[b]);
     }
+  } else if (warp >= kKeyWarp0) {
+    // ---- kept keys (kcopy): K_out rows of this CTA's kept rows of every unit,
+    // K[token], copied while the pipeline runs.  Nothing waits for them and
+    // they wait for nothing (the keep list and K are complete at launch); each
+    // warp takes every other pair of rows, a half-warp a 256-byte row.
+    if (kcopy) {
+      const int c = lane & 15;
+      const int rsub = 2 * (warp - kKeyWarp0) + (lane >> 4);   // 0..3
+      // batch q: rows 4 (16 (q % 2) + i) + rsub of unit q / 2's tile, i < 16;
+      // the next batch's tokens load while this batch's rows are in flight
+      auto load_tok = [&](int q, int (&tk)[16]) {
+        const Unit& d = sm.unit[q >> 1];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int rr = 4 * (16 * (q & 1) + i) + rsub;
+          tk[i] = rr < d.rows ? __ldg(keep_idx + d.orow + rr) : -1;
+        }
+      };
+      int tok[16];
+      if (nunits > 0) load_tok(0, tok);
+#pragma unroll 1
+      for (int q = 0; q < 2 * nunits; ++q) {
+        const Unit d = sm.unit[q >> 1];
+        const int h = q & 1;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int rr = 4 * (16 * h + i) + rsub;
+          if (rr < d.rows && (tok[i] < 0 || tok[i] >= d.n)) {
+            if (c == 0) set_status(tb.status, VC_ERR_DEVICE_INDEX);
+            tok[i] = -1;
+          }
+        }
+        const uint4* Kt = K + (int64_t)d.kv_row * 16 + c;
+        uint4 kv[16];
+        uint32_t have = 0;
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (tok[i] >= 0) {
+            kv[i] = __ldg(Kt + (int64_t)tok[i] * 16);
+            have |= 1u << i;
+          }
+        if (q + 1 < 2 * nunits) load_tok(q + 1, tok);
+        uint4* Ko = K_out + d.orow * 16 + c;
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if ((have >> i) & 1u) Ko[(int64_t)(4 * (16 * h + i) + rsub) * 16] = kv[i];
+      }
+    }
   } else if (warp >= kEpiWarp0) {
     // ---- epilogue: V_out = mu V_k + (1 - mu) O / lsum (V_k when nothing is dropped)
     const int q4 = warp & 3;                          // TMEM lane quadrant of this warp
@@ -628,14 +681,14 @@ int fuse_tcp_pairs() {
 
 cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const Tables& tb,
                            const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
-                           void* K_out, void* V_out, void* Vs, int64_t vs_rows, int units_gather,
-                           int units, cudaStream_t st) {
+                           void* K_out, void* V_out, void* Vs, int64_t vs_rows, bool kcopy,
+                           int units_gather, int units, cudaStream_t st) {
   if (units_gather == 0) return cudaSuccess;
   {
-    ProfileScope ps("gather_kv", st);
+    ProfileScope ps(kcopy ? "gather_v" : "gather_kv", st);
     gather_kv_kernel<<<units_gather, kGatherThreads, 0, st>>>(
         static_cast<const uint4*>(K), static_cast<const uint4*>(V), sh, tb, keep_idx, drop_idx,
-        static_cast<uint4*>(K_out), static_cast<uint4*>(Vs));
+        static_cast<uint4*>(K_out), static_cast<uint4*>(Vs), kcopy ? 0 : 1);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -656,8 +709,9 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
   for (int64_t o = 0; o < units; o += per_launch) {
     const int cnt = (int)std::min<int64_t>(per_launch, units - o);
     const int p = std::min(pairs, cnt);
-    pf::fuse_v_tcp_kernel<<<2 * p, pf::kThreads, smem, st>>>(m128, m64, sh, tb, units, (int)o, cnt, mu,
-                                                             kLog2e / tau, static_cast<__nv_bfloat16*>(V_out));
+    pf::fuse_v_tcp_kernel<<<2 * p, pf::kThreads, smem, st>>>(
+        m128, m64, sh, tb, units, (int)o, cnt, mu, kLog2e / tau, static_cast<__nv_bfloat16*>(V_out),
+        kcopy ? 1 : 0, keep_idx, static_cast<const uint4*>(K), static_cast<uint4*>(K_out));
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

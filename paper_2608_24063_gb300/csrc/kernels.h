@@ -40,14 +40,16 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
                             const TcPlan& tp, float2* part, float* nlse_pad, const float* lse_nat,
                             float* scores, cudaStream_t st);
 
-// bf16, d = 128: K_out = K[keep] and the survivors' values compacted into Vs
-// (gather), then V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on tcgen05.
+// bf16, d = 128: the survivors' values compacted into Vs (gather), then
+// V_out = mu V_k + (1-mu) softmax(V_k V_d^T / tau) V_d on tcgen05.  K_out =
+// K[keep] is copied by the fusion's own key warps (kcopy: K in device memory)
+// or else by the gather.
 int fuse_rows_per_tile_tc();
 int gather_rows_per_block();
 cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const Tables& tb,
                            const int32_t* keep_idx, const int32_t* drop_idx, float mu, float tau,
-                           void* K_out, void* V_out, void* Vs, int64_t vs_rows, int units_gather,
-                           int units, cudaStream_t st);
+                           void* K_out, void* V_out, void* Vs, int64_t vs_rows, bool kcopy,
+                           int units_gather, int units, cudaStream_t st);
 
 // Ranking (sorted 1024-key chunks, `chunks`: kSortChunk keys per chunk,
 // Req::chunk0 locates a request's chunks) and ascending keep/drop compaction.

@@ -125,21 +125,22 @@ KERNEL_WORK = {
 }
 
 
-def traffic_for(kernel):
-    """dram bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+def traffic_for(kernel, workload):
+    """dram bytes per launch from the committed ncu summary: only for the workload
+    it was captured on, and only while the kernel's source is unchanged."""
     path = os.path.join(ROOT, "profiles", "traffic.md")
-    if not os.path.exists(path):
+    if workload is None or not os.path.exists(path):
         return None
     for line in open(path):
         cells = [c.strip() for c in line.strip().strip("|").split("|")]
-        if len(cells) != 4 or cells[0] != kernel:
+        if len(cells) != 5 or cells[0] != kernel or cells[1] != workload:
             continue
-        src = os.path.join(ROOT, cells[1])
+        src = os.path.join(ROOT, cells[2])
         if not os.path.exists(src):
             return None
         with open(src, "rb") as f:
             digest = hashlib.sha256(f.read()).hexdigest()[:16]
-        return int(cells[3]) if digest == cells[2] else None
+        return int(cells[4]) if digest == cells[3] else None
     return None
 
 
@@ -588,7 +589,7 @@ def run_decode(args):
         "kernels_ms_per_step": kern,
         "roofline": {"kernel": main_kernel, "bound": "hbm", "achieved": achieved,
                      "peak": pk["hbm"], "unit": "GB/s", "frac": achieved / pk["hbm"],
-                     "traffic": traffic_for(main_kernel),
+                     "traffic": traffic_for(main_kernel, "decode, %d requests" % n_req),
                      "peak_source": pk["source"]},
         "cpu_baseline": {"value": cpu, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
                          "sample": "%d single-request steps over all %d layers (fp64 numpy)" % (nr, L)},
@@ -887,7 +888,10 @@ def main():
     value = job_value(job_units, ms_step)
     pk = peaks()
 
-    # dominant kernel
+    # dominant kernel; its DRAM traffic was captured for the default options on one GPU
+    default_opts = (world == 1 and args.schedule == "parabola" and args.drop == "survivors"
+                    and args.rank == "shared")
+    traffic_wl = "workload %d" % args.workload if default_opts else None
     dom = max(kern.items(), key=lambda kv: kv[1][0]) if kern else None
     roof = None
     if dom:
@@ -897,12 +901,12 @@ def main():
         if kind == "tensor":
             ach = work[key] / per / 1e12
             roof = {"kernel": name, "bound": "tensor", "achieved": ach, "peak": pk["tc"],
-                    "unit": "TFLOP/s", "frac": ach / pk["tc"], "traffic": traffic_for(name),
+                    "unit": "TFLOP/s", "frac": ach / pk["tc"], "traffic": traffic_for(name, traffic_wl),
                     "peak_source": pk["source"] + " bf16 dense burst"}
         else:
             ach = work[key] / per / 1e9
             roof = {"kernel": name, "bound": "hbm", "achieved": ach, "peak": pk["hbm"],
-                    "unit": "GB/s", "frac": ach / pk["hbm"], "traffic": traffic_for(name),
+                    "unit": "GB/s", "frac": ach / pk["hbm"], "traffic": traffic_for(name, traffic_wl),
                     "peak_source": pk["source"] + " copy bandwidth"}
     t_hbm = work["bytes"] / (pk["hbm"] * 1e9)
     t_tc = work["flops_score"] / (pk["tc"] * 1e12)

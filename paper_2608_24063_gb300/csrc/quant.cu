@@ -19,6 +19,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "kernels.h"
 #include "profile.h"
 #include "vc_common.cuh"
@@ -49,6 +51,31 @@ __device__ __forceinline__ uint32_t code_of(float x, float lo, float scale, floa
   float t = __fmul_rn(a, inv);
   if (fabsf(t - floorf(t) - 0.5f) < 1e-5f || !(fabsf(t) <= 16.f)) t = __fdiv_rn(a, scale);
   return (uint32_t)fminf(fmaxf(rintf(t), 0.f), 15.f);
+}
+
+// Two codes with packed fp32 pairs, the same decision as code_of: t is
+// rounded to nearest-even by adding 1.5 * 2^23 (exact for 0 <= t < 2^22, the
+// integer then sits in the low bits of the sum); a code whose t lies within
+// 1e-5 of a half-integer (|t - rint(t)| > 0.5 - 1e-5), outside [0, 16] or is
+// NaN, or whose scale is not positive, is decided by code_of instead.
+constexpr float kRound = 12582912.f;                 // 1.5 * 2^23
+constexpr uint32_t kRoundBits = 0x4B400000u;
+__device__ __forceinline__ void codes2(float2 x, float2 lo, float2 scale, float2 inv, uint32_t& q0,
+                                       uint32_t& q1) {
+  const float2 a = __fadd2_rn(x, make_float2(-lo.x, -lo.y));
+  const float2 t = __fmul2_rn(a, inv);
+  const float2 r = __fadd2_rn(t, make_float2(kRound, kRound));
+  const float2 n = __fadd2_rn(r, make_float2(-kRound, -kRound));
+  const float2 e = __fadd2_rn(t, make_float2(-n.x, -n.y));
+  const bool f0 = scale.x > 0.f && t.x >= 0.f && t.x <= 16.f && fabsf(e.x) <= 0.5f - 1e-5f;
+  const bool f1 = scale.y > 0.f && t.y >= 0.f && t.y <= 16.f && fabsf(e.y) <= 0.5f - 1e-5f;
+  q0 = f0 ? min(__float_as_uint(r.x) - kRoundBits, 15u) : code_of(x.x, lo.x, scale.x, inv.x);
+  q1 = f1 ? min(__float_as_uint(r.y) - kRoundBits, 15u) : code_of(x.y, lo.y, scale.y, inv.y);
+}
+
+// Elementwise minimum and maximum of bf16 pairs (exact: no rounding).
+__device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t u) {
+  return *reinterpret_cast<const __nv_bfloat162*>(&u);
 }
 
 struct GroupRows {
@@ -138,20 +165,55 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
   const int lane = threadIdx.x & 31, c0 = lane * CPT;
   const GroupRows gr = group_rows(tb, unit);
   const T* kp = K + gr.row * D + c0;
+  constexpr bool kBf16 = std::is_same<T, __nv_bfloat16>::value;
   float mn[CPT], mx[CPT];
+  if constexpr (kBf16) {
+    // per-channel minimum and maximum on bf16 pairs
+    __nv_bfloat162 lo2[CPT / 2], hi2[CPT / 2];
 #pragma unroll
-  for (int j = 0; j < CPT; ++j) {
-    mn[j] = INFINITY;
-    mx[j] = -INFINITY;
-  }
+    for (int j = 0; j < CPT / 2; ++j) {
+      lo2[j] = __floats2bfloat162_rn(INFINITY, INFINITY);
+      hi2[j] = __floats2bfloat162_rn(-INFINITY, -INFINITY);
+    }
 #pragma unroll 8
-  for (int i = 0; i < gr.nrows; ++i) {
-    float v[CPT];
-    load_cpt<T, CPT>(kp + i * D, v);
+    for (int i = 0; i < gr.nrows; ++i) {
+      uint32_t w[CPT / 2];
+      if constexpr (CPT == 4) {
+        const uint2 u = *reinterpret_cast<const uint2*>(kp + i * D);
+        w[0] = u.x;
+        w[CPT / 2 - 1] = u.y;
+      } else {
+        w[0] = *reinterpret_cast<const uint32_t*>(kp + i * D);
+      }
+#pragma unroll
+      for (int j = 0; j < CPT / 2; ++j) {
+        lo2[j] = __hmin2(lo2[j], as_bf162(w[j]));
+        hi2[j] = __hmax2(hi2[j], as_bf162(w[j]));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < CPT / 2; ++j) {
+      const float2 l = __bfloat1622float2(lo2[j]), h = __bfloat1622float2(hi2[j]);
+      mn[2 * j] = l.x;
+      mn[2 * j + 1] = l.y;
+      mx[2 * j] = h.x;
+      mx[2 * j + 1] = h.y;
+    }
+  } else {
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
-      mn[j] = fminf(mn[j], v[j]);
-      mx[j] = fmaxf(mx[j], v[j]);
+      mn[j] = INFINITY;
+      mx[j] = -INFINITY;
+    }
+#pragma unroll 8
+    for (int i = 0; i < gr.nrows; ++i) {
+      float v[CPT];
+      load_cpt<T, CPT>(kp + i * D, v);
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) {
+        mn[j] = fminf(mn[j], v[j]);
+        mx[j] = fmaxf(mx[j], v[j]);
+      }
     }
   }
   float ks[CPT], ki[CPT];
@@ -168,7 +230,9 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
     load_cpt<T, CPT>(kp + i * D, v);
     uint32_t q[CPT];
 #pragma unroll
-    for (int j = 0; j < CPT; ++j) q[j] = code_of(v[j], mn[j], ks[j], ki[j]);
+    for (int j = 0; j < CPT; j += 2)
+      codes2(make_float2(v[j], v[j + 1]), make_float2(mn[j], mn[j + 1]), make_float2(ks[j], ks[j + 1]),
+             make_float2(ki[j], ki[j + 1]), q[j], q[j + 1]);
     store_codes<CPT>(kc + i * (D / 2), q);
   }
   // values: lane (row i, 32-channel group gv) takes the group whole (NG groups
@@ -179,18 +243,44 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
   for (int i = lane / NG; i < gr.nrows; i += RPP) {
     float v[kGroup];
     const T* src = V + (gr.row + i) * D + gv * kGroup;
+    float lo, hi;
+    if constexpr (kBf16) {
+      // the group's 32 values as 16 bf16 pairs: minimum and maximum on pairs
+      uint32_t w[kGroup / 2];
 #pragma unroll
-    for (int k = 0; k < kGroup; k += CPT) {
-      float u[CPT];
-      load_cpt<T, CPT>(src + k, u);
+      for (int k = 0; k < kGroup / 2; k += 4) {
+        const uint4 u = *reinterpret_cast<const uint4*>(src + 2 * k);
+        w[k] = u.x; w[k + 1] = u.y; w[k + 2] = u.z; w[k + 3] = u.w;
+      }
+      __nv_bfloat162 l2 = as_bf162(w[0]), h2 = as_bf162(w[0]);
 #pragma unroll
-      for (int j = 0; j < CPT; ++j) v[k + j] = u[j];
-    }
-    float lo = v[0], hi = v[0];
+      for (int k = 1; k < kGroup / 2; ++k) {
+        l2 = __hmin2(l2, as_bf162(w[k]));
+        h2 = __hmax2(h2, as_bf162(w[k]));
+      }
+      const float2 lf = __bfloat1622float2(l2), hf = __bfloat1622float2(h2);
+      lo = fminf(lf.x, lf.y);
+      hi = fmaxf(hf.x, hf.y);
 #pragma unroll
-    for (int k = 1; k < kGroup; ++k) {
-      lo = fminf(lo, v[k]);
-      hi = fmaxf(hi, v[k]);
+      for (int k = 0; k < kGroup / 2; ++k) {
+        v[2 * k] = __uint_as_float(w[k] << 16);
+        v[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < kGroup; k += CPT) {
+        float u[CPT];
+        load_cpt<T, CPT>(src + k, u);
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) v[k + j] = u[j];
+      }
+      lo = v[0];
+      hi = v[0];
+#pragma unroll
+      for (int k = 1; k < kGroup; ++k) {
+        lo = fminf(lo, v[k]);
+        hi = fmaxf(hi, v[k]);
+      }
     }
     const float vs = __fdiv_rn(__fsub_rn(hi, lo), 15.f);
     const float vi = vs > 0.f ? __frcp_rn(vs) : 0.f;
@@ -200,7 +290,12 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_kernel(
     for (int b = 0; b < 4; ++b) {
       w[b] = 0u;
 #pragma unroll
-      for (int k = 0; k < 8; ++k) w[b] |= code_of(v[8 * b + k], lo, vs, vi) << (4 * k);
+      for (int k = 0; k < 8; k += 2) {
+        uint32_t q0, q1;
+        codes2(make_float2(v[8 * b + k], v[8 * b + k + 1]), make_float2(lo, lo), make_float2(vs, vs),
+               make_float2(vi, vi), q0, q1);
+        w[b] |= (q0 << (4 * k)) | (q1 << (4 * k + 4));
+      }
     }
     *reinterpret_cast<uint4*>(Vc + (gr.row + i) * (D / 2) + gv * (kGroup / 2)) = make_uint4(w[0], w[1], w[2], w[3]);
   }

@@ -279,6 +279,31 @@ def test_values_in_host_memory(kernel_path):
     assert torch.equal(i1, i2) and torch.equal(Ko1, Ko2) and torch.equal(Vo1, Vo2)
 
 
+def test_keys_and_values_in_host_memory(kernel_path):
+    # the fusion step with K and V in pinned host memory: the kept keys are then
+    # copied by the gather (the tensor-core fusion copies them itself only from
+    # device memory); same bits as from HBM
+    L, Hq, Hkv, d, n, W = 3, 8, 2, 128, 1500, 16
+    Q = _rand((L, Hq, W, d), 9201, torch.bfloat16).to(DEV)
+    K = _rand((L, Hkv, n, d), 9202, torch.bfloat16)
+    V = _rand((L, Hkv, n, d), 9203, torch.bfloat16)
+    hK, hV = K.pin_memory(), V.pin_memory()
+    if not (vc.viscache_device_accessible(hK) and vc.viscache_device_accessible(hV)):
+        pytest.skip("pinned host memory is not mapped into the device's address space here")
+    B, Nq, _ = vc.viscache_plan_budgets(L, n, 23, 100)
+    s = vc.prunekv_score(Q, K.to(DEV))
+    _, keep, drop = vc.prunekv_select(s, B, Nq)
+    Ko1, Vo1 = vc.prunekv_fuse_compact(K.to(DEV), V.to(DEV), B, Nq, keep, drop, 0.7, 1.0)
+    # outputs and workspace on the device (the binding would put them beside K)
+    Ko2 = torch.empty_like(Ko1)
+    Vo2 = torch.empty_like(Vo1)
+    ws = torch.empty(vc.prunekv_fuse_workspace_size(B, Hkv, d, n, Nq), dtype=torch.uint8, device=DEV)
+    vc.prunekv_fuse_compact(hK, hV, B, Nq, keep, drop, 0.7, 1.0, K_out=Ko2, V_out=Vo2, ws=ws)
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+    torch.cuda.synchronize()
+    assert torch.equal(Ko1, Ko2) and torch.equal(Vo1, Vo2)
+
+
 def test_generator_same_bits_on_device():
     wl = synth.scaled(synth.WORKLOADS[3], "slice", L=2)
     q_cpu = synth.make_q(wl, 0, "cpu")

@@ -2,18 +2,19 @@
 // Eq. (weight_fusion), Algorithm 1 step 3.
 //
 // gather_kv_kernel (HBM-bound copy): for every (request, layer, KV head) the
-//   kept key rows go to K_out (bit-exact), and the survivors' value rows --
-//   kept then dropped, each list in ascending position -- are compacted into a
-//   dense workspace slab Vs, so the fusion can stream them with TMA.
+//   survivors' value rows -- kept then dropped, each list in ascending
+//   position -- are compacted into a dense workspace slab Vs, so the fusion
+//   can stream them with TMA; the kept key rows go to K_out (bit-exact) here
+//   only when K is not in device memory (else the fusion copies them).
 // fuse_v_tcp_kernel: persistent CTA pairs, each taking a share of the units
 //   (request, layer, KV head, 256 kept rows) in turn:
 //   O = softmax_row(V_k V_d^T / tau) V_d online over tiles of 128 dropped rows,
 //   V_out = mu V_k + (1 - mu) O, on 2-SM tcgen05.mma with fp32 accumulators in
 //   tensor memory; the numerators P go from the softmax warps to the second
-//   product through tensor memory.  Warp roles (448 threads, one CTA per SM):
+//   product through tensor memory.  Warp roles (512 threads, one CTA per SM):
 //   warps 0-7 softmax, warp 8 TMA and the tensor-memory allocation, one
-//   thread of warp 9 (even CTA) the MMAs, warps 10-13 the epilogue.  Every
-//   wait is bounded (tc_common.cuh).
+//   thread of warp 9 (even CTA) the MMAs, warps 10-13 the epilogue, warps
+//   14-15 the kept-key copy.  Every wait is bounded (tc_common.cuh).
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -126,7 +127,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // CTA), 10-13 the epilogue: once O[k % 2] is final it reads O, the row sums
 // and V_k, writes mu V_k + (1 - mu) O / lsum in bf16 through a staging buffer,
 // and frees O[k % 2] and vk[k % 2] -- while the MMAs and the softmax of unit
-// k + 1 go on.
+// k + 1 go on; 14-15 copy the CTA's kept keys of every unit into K_out.
 //
 // Every barrier completes once per unit (or per tile) and no waiter can fall
 // two phases behind: the loader refills vk[b] only after the epilogue freed it,

@@ -109,8 +109,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // ---------------------------------------------------------------------------
 // persistent fusion: one CTA pair per TPC for the whole launch
 //
-// Same arithmetic as fuse_v_tc_kernel, organised so that nothing waits at a
-// unit boundary.  The launch holds as many pairs as fit at once (one CTA per
+// Organised so that nothing waits at a unit boundary.  The launch holds as many pairs as fit at once (one CTA per
 // SM: 512 tensor-memory columns and ~214 KB of shared memory each); pair p
 // takes the units p, p + P, p + 2P, ... of the list ordered longest first.
 // Tensor memory per CTA: O[0] [0,128), O[1] [128,256) -- unit k accumulates
@@ -120,7 +119,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 // S, K = 128 for O: 16 MMAs and 2-3 commits per tile).  The issue order is
 // S(t), O(t-1), so S(t) runs while the softmax works on tile t-1.
 //
-// Warps: 0-7 softmax (as in fuse_v_tc_kernel, 64 columns each), 8 the
+// Warps: 0-7 softmax (two per TMEM lane quadrant, 64 columns each), 8 the
 // producer (lane 0 issues the TMA loads: the unit's kept rows into vk[k % 2],
 // then its dropped tiles into a 3-stage ring; lane 1 tells the even CTA when
 // this CTA's kept rows of each unit have landed), 9 the MMA issuer (even
@@ -546,7 +545,7 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
       if (ok) {
         tc_fence_after();
         const bool have_o = d.D > 0;
-        const float lt = sm.lsum[b][q4][0][lane] + sm.lsum[b][q4][1][lane];   // same order as fuse_v_tc
+        const float lt = sm.lsum[b][q4][0][lane] + sm.lsum[b][q4][1][lane];
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.lsum_empty[b]);
         const float w_o = have_o ? (1.f - mu) / lt : 0.f;

@@ -232,13 +232,17 @@ int prunekv_select(const float* scores, int32_t L, int32_t Hkv, int32_t n_vis,
  *   V_out = mu * V_k + (1 - mu) * Phi V_d,  Phi = row-softmax(V_k V_d^T / tau)
  *           -- Eq. (redistribution), Eq. (weight_fusion); V_out = V_k when the
  *           drop set is empty.  fp32 arithmetic, rounded to dtype (RNE).
- *   K, V              device [L][Hkv][n][d], dtype
+ *   K, V              [L][Hkv][n][d], dtype: device memory, or host memory the
+ *                     device can read (viscache_device_accessible == 1; only the
+ *                     kept rows of K and the survivors' rows of V are read)
  *   B, Nq             HOST budgets as for prunekv_select
  *   keep_idx/drop_idx device lists from prunekv_select
  *   mu in [0, 1], tau > 0
  *   K_out, V_out      device, dense varlen (rows Hkv * sum_l B_l, d columns)
  *   ws                workspace of prunekv_fuse_workspace_size(B, L, Hkv, d, n, Nq) bytes
- *                     (bf16, d = 128 also compacts the survivors' values there)
+ *                     (bf16, d = 128 also compacts the survivors' values there;
+ *                     the tensor-core fusion then copies K_out itself while its
+ *                     products run when K is device memory)
  */
 size_t prunekv_fuse_workspace_size(const int32_t* B, int32_t L, int32_t Hkv, int32_t d,
                                    int32_t n_vis, int32_t Nq);

@@ -19,7 +19,9 @@ request and every (layer, KV head):
 The counts of checked (layer, KV head) sets are asserted: 480 for the 72B shape
 (h = 60 layers with B_l > 0, 8 KV heads) and 8 x 21 x 4 = 672 for the batch.
 The batch launch also equals, bit for bit, the same requests compressed one at
-a time, and repeated launches of the batch are bit-identical.
+a time, and repeated launches of the batch are bit-identical.  Three 72B-shaped
+requests in one call (more fusion units than one persistent launch holds)
+equal the requests compressed alone, with sampled sets against the oracle.
 """
 from fractions import Fraction
 
@@ -194,3 +196,69 @@ def test_repeated_launches_bit_identical():
         assert torch.equal(idx, idx0), "launch %d idx" % rep
         assert torch.equal(Ko, Ko0), "launch %d K_out" % rep
         assert torch.equal(Vo, Vo0), "launch %d V_out" % rep
+
+
+def test_fusion_across_launches_equals_single_requests():
+    """Three 72B-shaped requests in one call: about 50,000 fusion units, more than
+    one launch of the persistent fusion takes (a pair holds at most 512 unit
+    descriptors), so the call runs the fusion in several launches.  Each
+    request's rows equal, bit for bit, the same request compressed alone (one
+    launch), and sampled (layer, KV head) sets -- the first and last kept layer,
+    the first and last KV head -- match the oracle's fusion on the GPU's own
+    keep and drop lists."""
+    from tests.parity import check_v_rows
+    wl = synth.replicated(synth.WORKLOADS[4], 3)
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16)
+    plans = [vc.viscache_plan_budgets(wl.L, r.n, r.rr_num, r.rr_den) for r in wl.requests]
+    units = sum(wl.Hkv * ((b + 255) // 256) for B, _, _ in plans for b in B if b > 0)
+    per_launch = torch.cuda.get_device_properties(0).multi_processor_count // 2 * 512
+    assert units > per_launch, (units, per_launch)
+    qs, ks, vs = synth.generate(wl, DEV)
+    shapes = [(q.shape, k.shape) for q, k in zip(qs, ks)]
+    Q = torch.cat([q.flatten() for q in qs])
+    K = torch.cat([k.flatten() for k in ks])
+    V = torch.cat([v.flatten() for v in vs])
+    del qs, ks, vs
+    Ko, Vo, idx = vc.prunekv_compress(_batch(wl), prm, Q, K, V)
+    torch.cuda.synchronize()
+    off_r = off_q = off_kv = 0
+    checked = 0
+    for i, r in enumerate(wl.requests):
+        qshape, kshape = shapes[i]
+        nq, nkv = int(np.prod(qshape)), int(np.prod(kshape))
+        q_i = Q[off_q:off_q + nq].view(qshape)
+        k_i = K[off_kv:off_kv + nkv].view(kshape)
+        v_i = V[off_kv:off_kv + nkv].view(kshape)
+        one = vc.Batch([r.n], [r.W], [(r.rr_num, r.rr_den)])
+        rows = vc.compressed_rows(one, prm)
+        ko, vo, ix = vc.prunekv_compress(one, prm, q_i, k_i, v_i)
+        torch.cuda.synchronize()
+        assert torch.equal(idx[off_r:off_r + rows], ix), "request %d idx" % i
+        assert torch.equal(Ko[off_r:off_r + rows], ko), "request %d K_out" % i
+        assert torch.equal(Vo[off_r:off_r + rows], vo), "request %d V_out" % i
+        del ko, vo, ix
+        B, Nq, h = plans[i]
+        s = vc.prunekv_score(q_i, k_i)
+        _, keep, drop = vc.prunekv_select(s, B, Nq)
+        torch.cuda.synchronize()
+        assert torch.equal(keep, idx[off_r:off_r + rows]), "request %d keep" % i
+        keep_c, drop_c = keep.cpu().numpy(), drop.cpu().numpy()
+        P = Qd = 0
+        for l in range(wl.L):
+            b = B[l]
+            D = Nq - b if b > 0 else 0
+            if b > 0 and l in (0, h - 1):
+                for g in (0, wl.Hkv - 1):
+                    kl = keep_c[wl.Hkv * P + g * b:wl.Hkv * P + (g + 1) * b]
+                    dl = drop_c[wl.Hkv * Qd + g * D:wl.Hkv * Qd + (g + 1) * D]
+                    ref = ok.fuse_values(np64(v_i[l, g].cpu()), kl, dl, MU, TAU)
+                    got = np64(Vo[off_r + wl.Hkv * P + g * b:off_r + wl.Hkv * P + (g + 1) * b].cpu())
+                    check_v_rows(got, ref, TOL[torch.bfloat16], "request %d layer %d head %d" % (i, l, g))
+                    checked += 1
+            P += b
+            Qd += D
+        off_r += rows
+        off_q += nq
+        off_kv += nkv
+    assert checked == 3 * 2 * 2
+    assert off_r == vc.compressed_rows(_batch(wl), prm)

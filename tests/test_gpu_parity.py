@@ -75,6 +75,22 @@ def test_compress_equals_step_api(case):
     assert torch.equal(idx, ref["keep"]) and torch.equal(Ko, ref["K_out"]) and torch.equal(Vo, ref["V_out"])
 
 
+def test_maximum_visual_tokens(kernel_path):
+    # n at its limit (65,536 visual tokens): scores, ranking, both lists, K_out
+    # and V_out against the oracle; the fused call equals the steps bit for bit
+    L, Hq, Hkv, d, n, W, rr = 2, 4, 2, 128, 65536, 16, (1, 10)
+    Q = _rand((L, Hq, W, d), 9301, torch.bfloat16)
+    K = _rand((L, Hkv, n, d), 9302, torch.bfloat16)
+    V = _rand((L, Hkv, n, d), 9303, torch.bfloat16)
+    B, Nq, h = vc.viscache_plan_budgets(L, n, *rr)
+    gpu = run_steps(Q.to(DEV), K.to(DEV), V.to(DEV), B, Nq)
+    check_request(Q, K, V, B, Nq, gpu, 0.7, 1.0)
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    Ko, Vo, idx = vc.prunekv_compress(vc.Batch([n], [W], [rr]), prm, Q.to(DEV), K.to(DEV), V.to(DEV))
+    torch.cuda.synchronize()
+    assert torch.equal(idx, gpu["keep"]) and torch.equal(Ko, gpu["K_out"]) and torch.equal(Vo, gpu["V_out"])
+
+
 def test_mu_one_is_plain_pruning_bit_exact():
     L, Hq, Hkv, d, n, W = 3, 4, 2, 128, 300, 8
     Q, K, V = (_rand(s, 700 + i, torch.bfloat16).to(DEV) for i, s in

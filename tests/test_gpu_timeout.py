@@ -115,3 +115,36 @@ def test_fused_pass_and_static_scoring_report_timeouts(inject):
     Ko, Vo, _ = out
     assert not bool(torch.isnan(Ko.float()).any()) and not bool(torch.isnan(Vo.float()).any())
 
+
+
+def test_abort_with_several_units_per_fusion_pair(inject):
+    # a shape whose fusion deals two to four units to every CTA pair and whose
+    # score passes run tens of tiles per unit: the injected give-ups then abort
+    # pairs in the middle of later units; the call returns, reports the
+    # timeout, and the context stays usable
+    L2, Hq2, Hkv2, n2, W2 = 8, 28, 4, 8192, 20
+    mk = lambda shape, k: synth._round(synth.normal(4200 + k, 0, int(np.prod(shape)), "cpu").view(*shape),
+                                        torch.bfloat16)
+    q, k, v = mk((L2, Hq2, W2, d), 1), mk((L2, Hkv2, n2, d), 2), mk((L2, Hkv2, n2, d), 3)
+    Q, K, V = q.to(DEV), k.to(DEV), v.to(DEV)
+    B, Nq, _ = vc.viscache_plan_budgets(L2, n2, *RR)
+    units = sum(Hkv2 * ((b + 255) // 256) for b in B if b > 0)
+    assert units > 2 * (torch.cuda.get_device_properties(0).multi_processor_count // 2), units
+    batch = vc.Batch([n2], [W2], [RR])
+    prm = vc.make_params(L2, Hq2, Hkv2, d, vc.VC_BF16)
+    ws = torch.empty(vc.prunekv_workspace_size(batch, prm), dtype=torch.uint8, device=DEV)
+    for mask in (vc.VC_TEST_WAIT_FUSE,
+                 vc.VC_TEST_WAIT_SCORE_LSE | vc.VC_TEST_WAIT_SCORE_COLSUM | vc.VC_TEST_WAIT_FUSE):
+        inject(mask)
+        t0 = time.perf_counter()
+        vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
+        assert vc.prunekv_get_status(ws) == vc.VC_ERR_DEVICE_TIMEOUT
+        assert time.perf_counter() - t0 < ABORT_SECONDS
+    inject(0)
+    vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+    s = vc.prunekv_score(Q, K)
+    _, keep, drop = vc.prunekv_select(s, B, Nq)
+    Ko, Vo = vc.prunekv_fuse_compact(K, V, B, Nq, keep, drop, 0.7, 1.0)
+    torch.cuda.synchronize()
+    check_request(q, k, v, B, Nq, dict(scores=s, keep=keep, drop=drop, K_out=Ko, V_out=Vo), 0.7, 1.0)

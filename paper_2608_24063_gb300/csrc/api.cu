@@ -227,21 +227,25 @@ struct Layout {
   // Copy the table image into the workspace and clear the status word.  Small
   // images (every single request and typical batches) travel as a kernel
   // parameter, so the upload is an ordinary launch on the stream (no host
-  // blocking, capturable in a CUDA graph); larger ones use one memcpy.
+  // blocking, capturable in a CUDA graph); larger ones use one memcpy, and
+  // then an upload of no bytes clears the status word, so that the kernels
+  // after it always follow a kernel (their dependent launches order
+  // themselves on the kernel before them).
   cudaError_t upload(uint8_t* ws, cudaStream_t st) const {
     const size_t bytes = table_end - table_begin;
+    int32_t* status = reinterpret_cast<int32_t*>(ws + o_status);
     if (bytes <= sizeof(TableImage::bytes)) {
       TableImage im;
       memset(&im, 0, sizeof(im));
       fill(im.bytes);
-      return launch_upload(im, (uint32_t)bytes, ws + table_begin,
-                           reinterpret_cast<int32_t*>(ws + o_status), st);
+      return launch_upload(im, (uint32_t)bytes, ws + table_begin, status, st);
     }
     std::vector<uint8_t> img(bytes, 0);
     fill(img.data());
-    cudaError_t e = cudaMemsetAsync(ws + o_status, 0, kAlign, st);
+    cudaError_t e = cudaMemcpyAsync(ws + table_begin, img.data(), bytes, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return e;
-    return cudaMemcpyAsync(ws + table_begin, img.data(), bytes, cudaMemcpyHostToDevice, st);
+    static const TableImage none = {};
+    return launch_upload(none, 0u, ws + table_begin, status, st);
   }
 
   void fill(uint8_t* img) const {

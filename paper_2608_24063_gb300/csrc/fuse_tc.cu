@@ -45,6 +45,8 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kv_kernel(
     const uint4* __restrict__ K, const uint4* __restrict__ V, Shape sh, Tables tb,
     const int32_t* __restrict__ keep_idx, const int32_t* __restrict__ drop_idx,
     uint4* __restrict__ K_out, uint4* __restrict__ Vs, int keys) {
+  dep_wait();                        // the keep and drop lists
+  if (threadIdx.x == 0) dep_launch();
   const int rl = upper_index(tb.unit0_gather, sh.n_req * sh.L, (int32_t)blockIdx.x);
   const int r = rl / sh.L, l = rl % sh.L;
   const Req rq = tb.req[r];
@@ -266,6 +268,9 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
     prefetch_tmap(&tmRows64);
     int t = 0, kl = 0;
     bool ok = true;
+    // the survivor slab is the output of the kernel just before this one
+    dep_wait();
+    dep_launch();
     for (int k = 0; ok && k < nunits; ++k) {
       const Unit d = sm.unit[k];
       const int b = k & 1;
@@ -479,8 +484,10 @@ fuse_v_tcp_kernel(const __grid_constant__ CUtensorMap tmRows128, const __grid_co
   } else if (warp >= kKeyWarp0) {
     // ---- kept keys (kcopy): K_out rows of this CTA's kept rows of every unit,
     // K[token], copied while the pipeline runs.  Nothing waits for them and
-    // they wait for nothing (the keep list and K are complete at launch); each
-    // warp takes every other pair of rows, a half-warp a 256-byte row.
+    // they wait for nothing: K is an input and the keep list was written two
+    // kernels back, so both are complete once this kernel is scheduled (they
+    // start while the gather drains); each warp takes every other pair of
+    // rows, a half-warp a 256-byte row.
     if (kcopy) {
       const int c = lane & 15;
       const int rsub = 2 * (warp - kKeyWarp0) + (lane >> 4);   // 0..3
@@ -686,10 +693,9 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
   if (units_gather == 0) return cudaSuccess;
   {
     ProfileScope ps(kcopy ? "gather_v" : "gather_kv", st);
-    gather_kv_kernel<<<units_gather, kGatherThreads, 0, st>>>(
-        static_cast<const uint4*>(K), static_cast<const uint4*>(V), sh, tb, keep_idx, drop_idx,
-        static_cast<uint4*>(K_out), static_cast<uint4*>(Vs), kcopy ? 0 : 1);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_dep(gather_kv_kernel, dim3(units_gather), dim3(kGatherThreads), 0, st,
+                               static_cast<const uint4*>(K), static_cast<const uint4*>(V), sh, tb, keep_idx,
+                               drop_idx, static_cast<uint4*>(K_out), static_cast<uint4*>(Vs), kcopy ? 0 : 1);
     if (e != cudaSuccess) return e;
   }
   if (units == 0) return cudaSuccess;
@@ -709,10 +715,9 @@ cudaError_t launch_fuse_tc(const void* K, const void* V, const Shape& sh, const 
   for (int64_t o = 0; o < units; o += per_launch) {
     const int cnt = (int)std::min<int64_t>(per_launch, units - o);
     const int p = std::min(pairs, cnt);
-    pf::fuse_v_tcp_kernel<<<2 * p, pf::kThreads, smem, st>>>(
-        m128, m64, sh, tb, units, (int)o, cnt, mu, kLog2e / tau, static_cast<__nv_bfloat16*>(V_out),
-        kcopy ? 1 : 0, keep_idx, static_cast<const uint4*>(K), static_cast<uint4*>(K_out));
-    e = cudaGetLastError();
+    e = launch_dep(pf::fuse_v_tcp_kernel, dim3(2 * p), dim3(pf::kThreads), smem, st, m128, m64, sh, tb, units,
+                   (int)o, cnt, mu, kLog2e / tau, static_cast<__nv_bfloat16*>(V_out), kcopy ? 1 : 0, keep_idx,
+                   static_cast<const uint4*>(K), static_cast<uint4*>(K_out));
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -7,6 +7,30 @@
 
 namespace vc {
 
+// Launches kernel on st so that it may be scheduled before the previous kernel
+// on the stream has completed (programmatic stream serialisation); the kernel
+// orders itself with dep_wait / dep_launch (vc_common.cuh).  Defining
+// VC_SERIAL_LAUNCH launches every kernel fully serialised instead.
+template <typename... P, typename... A>
+cudaError_t launch_dep(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       A&&... args) {
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = at;
+#ifdef VC_SERIAL_LAUNCH
+  cfg.numAttrs = 0;
+#else
+  cfg.numAttrs = 1;
+#endif
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
+}
+
 // Plan-table image passed by value (kernel parameters may hold up to 32 KB).
 struct TableImage {
   alignas(16) uint8_t bytes[24 * 1024];

@@ -113,25 +113,6 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
   P1Smem& sm = *reinterpret_cast<P1Smem*>(align1024(smem_raw));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_rank();
-  const int unit = (int)(blockIdx.x >> 1);
-
-  const int r = upper_index(tb.unit0_tc1, sh.n_req, (int32_t)unit);
-  const Req rq = tb.req[r];
-  int u = unit - tb.unit0_tc1[r];
-  const int s = u % S;
-  u /= S;
-  const int rbp = u % rq.nrb;
-  u /= rq.nrb;
-  const int g = u % sh.Hkv, l = u / sh.Hkv;
-  const int rows = sh.G * rq.W;
-  const int ntiles_all = (rq.n + (int)kPairKeys - 1) / (int)kPairKeys;
-  const int tps = (ntiles_all + S - 1) / S;
-  const int t_begin = s * tps;
-  const int ntiles = max(0, min(ntiles_all, t_begin + tps) - t_begin);
-  const int qrow = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + rbp * 256 +
-                   (int)rank * (int)kTile;
-  const int krow0 = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + (int)rank * (int)kTile;
-
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
     for (int i = 0; i < kStagesPair; ++i) { mbar_init(&sm.k_full[i], 1); mbar_init(&sm.k_empty[i], 1); }
@@ -153,6 +134,26 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
   tc_fence_after();
   const uint32_t tbase = sm.tmem_base;
   volatile int* abort = &sm.abort;
+  // the plan tables come from the kernel just before this one
+  dep_wait();
+  if (threadIdx.x == 0) dep_launch();
+  const int unit = (int)(blockIdx.x >> 1);
+  const int r = upper_index(tb.unit0_tc1, sh.n_req, (int32_t)unit);
+  const Req rq = tb.req[r];
+  int u = unit - tb.unit0_tc1[r];
+  const int s = u % S;
+  u /= S;
+  const int rbp = u % rq.nrb;
+  u /= rq.nrb;
+  const int g = u % sh.Hkv, l = u / sh.Hkv;
+  const int rows = sh.G * rq.W;
+  const int ntiles_all = (rq.n + (int)kPairKeys - 1) / (int)kPairKeys;
+  const int tps = (ntiles_all + S - 1) / S;
+  const int t_begin = s * tps;
+  const int ntiles = max(0, min(ntiles_all, t_begin + tps) - t_begin);
+  const int qrow = (int)(rq.q_off / 128 + ((int64_t)l * sh.Hq + g * sh.G) * rq.W) + rbp * 256 +
+                   (int)rank * (int)kTile;
+  const int krow0 = (int)(rq.kv_off / 128 + ((int64_t)l * sh.Hkv + g) * rq.n) + (int)rank * (int)kTile;
 
   if (warp == kProducerWarp && lane == 0) {
     // ---- TMA producer (both CTAs): own rows and key halves, counted on the even CTA's barriers
@@ -334,6 +335,8 @@ score_lse_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 
 __global__ void lse_merge_kernel(Shape sh, Tables tb, int S, const float2* __restrict__ part,
                                  const float* __restrict__ lse_nat, float* __restrict__ nlse) {
+  dep_wait();                                 // the partial statistics of pass 1
+  if (threadIdx.x == 0) dep_launch();
   const Req rq = tb.req[blockIdx.y];
   const int rows = rq.C * rq.cw;              // padded rows of one (layer, KV head)
   const int64_t per = (int64_t)sh.L * sh.Hkv * rows;
@@ -494,7 +497,7 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
     int k_issued = 0, q_issued = 0;
-    bool ok = true;
+    bool ok = true, waited = false;
     for (int l = 0; ok && l < Ls; ++l) {
       const int ks = l & 1;
       if (!mbar_wait(&sm.k_empty[ks], ((l >> 1) & 1) ^ 1, abort)) break;
@@ -513,11 +516,22 @@ score_colsum_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_con
         const uint32_t q_full0 = map_to_rank(smem_u32(&sm.q_full[qs]), 0);
         tma_load_2d_pair(sm.q[qs][0], &tmQ, 0, qy0 + c * cw, q_full0);
         tma_load_2d_pair(sm.q[qs][1], &tmQ, 64, qy0 + c * cw, q_full0);
+        if (!waited) {
+          // the keys and the first rows are inputs and load while the
+          // kernel before this one drains; the normalisers are its output
+          dep_wait();
+          dep_launch();
+          waited = true;
+        }
         mbar_arrive_expect_tx(&sm.nl_full[qs], (uint32_t)cw * 4);
         bulk_load(sm.nlse[qs], nlse + rq.lsep_off + ((int64_t)(l * sh.Hkv + g) * C2 + c) * cw,
                   (uint32_t)cw * 4, &sm.nl_full[qs]);
         ++q_issued;
       }
+    }
+    if (!waited) {                 // no chunk (nothing scored, or an abort)
+      dep_wait();
+      dep_launch();
     }
     // every copy this CTA started has landed before the pair may leave: the
     // normalisers on this CTA's barriers, the tiles on the even CTA's
@@ -759,23 +773,22 @@ cudaError_t launch_score_tc(const void* Qw, const void* K, const Shape& sh, cons
     e = cudaFuncSetAttribute(score_lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
     if (e != cudaSuccess) return e;
     ProfileScope ps("score_lse_tc", st);
-    score_lse_tc_kernel<<<2 * tp.units1, kThreads, smem1, st>>>(mq, mk, sh, tb, tp.S, part, nlse_pad);
-    e = cudaGetLastError();
+    e = launch_dep(score_lse_tc_kernel, dim3(2 * tp.units1), dim3(kThreads), smem1, st, mq, mk, sh, tb, tp.S,
+                   part, nlse_pad);
     if (e != cudaSuccess) return e;
   }
   if (lse_nat || tp.S > 1) {
     ProfileScope ps("lse_merge", st);
-    lse_merge_kernel<<<dim3((unsigned)((tp.max_prows + 255) / 256), sh.n_req), 256, 0, st>>>(
-        sh, tb, tp.S, part, lse_nat, nlse_pad);
-    e = cudaGetLastError();
+    e = launch_dep(lse_merge_kernel, dim3((unsigned)((tp.max_prows + 255) / 256), sh.n_req), dim3(256), 0, st,
+                   sh, tb, tp.S, static_cast<const float2*>(part), lse_nat, nlse_pad);
     if (e != cudaSuccess) return e;
   }
   const size_t smem2 = sizeof(P2Smem) + 1024;
   e = cudaFuncSetAttribute(score_colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
   if (e != cudaSuccess) return e;
   ProfileScope ps("score_colsum_tc", st);
-  score_colsum_tc_kernel<<<2 * tp.units2, kThreads, smem2, st>>>(mq, mk, sh, tb, nlse_pad, scores);
-  return cudaGetLastError();
+  return launch_dep(score_colsum_tc_kernel, dim3(2 * tp.units2), dim3(kThreads), smem2, st, mq, mk, sh, tb,
+                    static_cast<const float*>(nlse_pad), scores);
 }
 
 }  // namespace vc

@@ -70,6 +70,8 @@ __global__ void __launch_bounds__(kSortChunk) chunk_sort_kernel(Shape sh, Tables
                                                                 const float* __restrict__ scores,
                                                                 uint64_t* __restrict__ chunks) {
   __shared__ uint64_t e[kSortChunk];
+  dep_wait();                                      // the scores
+  if (threadIdx.x == 0) dep_launch();
   Req rq;
   int64_t off, base;
   int nchunks;
@@ -107,6 +109,8 @@ __global__ void __launch_bounds__(kSortChunk) chunk_rank_kernel(Shape sh, Tables
                                                                 const uint64_t* __restrict__ chunks,
                                                                 int32_t* __restrict__ rank) {
   extern __shared__ uint64_t other[];               // [kRankGroup][kSortChunk]
+  dep_wait();                                      // the sorted chunks
+  if (threadIdx.x == 0) dep_launch();
   Req rq;
   int64_t off, base;
   int nchunks;
@@ -149,6 +153,8 @@ __global__ void __launch_bounds__(kScanThreads) compact_kernel(Shape sh, Tables 
                                                                int32_t* __restrict__ drop_idx) {
   constexpr int kWarps = kScanThreads / 32;
   __shared__ int32_t wk[kWarps], wd[kWarps], tot[2];
+  dep_wait();                                // the ranks
+  if (threadIdx.x == 0) dep_launch();
   const int g = blockIdx.y;
   const int rl = blockIdx.x;                 // request * L + layer
   const int r = rl / sh.L, l = rl % sh.L;
@@ -227,7 +233,8 @@ cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int
   const dim3 grid((unsigned)max_chunks, (unsigned)n_problems);
   {
     ProfileScope ps("chunk_sort", st);
-    chunk_sort_kernel<<<grid, kSortChunk, 0, st>>>(sh, tb, scores, chunks);
+    cudaError_t el = launch_dep(chunk_sort_kernel, grid, dim3(kSortChunk), 0, st, sh, tb, scores, chunks);
+    if (el != cudaSuccess) return el;
   }
   cudaError_t e0 = cudaGetLastError();
   if (e0 != cudaSuccess) return e0;
@@ -236,14 +243,17 @@ cudaError_t launch_select(const Shape& sh, const Tables& tb, int n_problems, int
     cudaError_t ea = cudaFuncSetAttribute(chunk_rank_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (ea != cudaSuccess) return ea;
     ProfileScope ps("chunk_rank", st);
-    chunk_rank_kernel<<<grid, kSortChunk, smem, st>>>(sh, tb, chunks, rank);
+    cudaError_t el = launch_dep(chunk_rank_kernel, grid, dim3(kSortChunk), smem, st, sh, tb,
+                                static_cast<const uint64_t*>(chunks), rank);
+    if (el != cudaSuccess) return el;
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   {
     ProfileScope ps("compact_keep_drop", st);
-    compact_kernel<<<dim3(sh.n_req * sh.L, sh.Hkv), kScanThreads, 0, st>>>(sh, tb, rank, keep_idx,
-                                                                           drop_idx);
+    cudaError_t el = launch_dep(compact_kernel, dim3(sh.n_req * sh.L, sh.Hkv), dim3(kScanThreads), 0, st,
+                                sh, tb, static_cast<const int32_t*>(rank), keep_idx, drop_idx);
+    if (el != cudaSuccess) return el;
   }
   return cudaGetLastError();
 }

@@ -8,6 +8,9 @@ namespace {
 
 __global__ void upload_kernel(const __grid_constant__ TableImage im, uint32_t bytes, uint8_t* dst,
                               int32_t* status) {
+  // launched fully serialised after everything before it on the stream; the
+  // kernels after it wait for it before they read the tables
+  dep_launch();
   const uint4* src = reinterpret_cast<const uint4*>(im.bytes);
   uint4* d = reinterpret_cast<uint4*>(dst);
   for (uint32_t i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = src[i];

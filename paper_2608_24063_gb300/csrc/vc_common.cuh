@@ -133,4 +133,22 @@ struct Kahan {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch.  The kernels after the first of a call are
+// launched with launch_dep (kernels.h), so each may be scheduled while the
+// kernel before it on the stream drains, and set up its shared and tensor
+// memory and read the inputs meanwhile.  dep_wait() returns once the previous
+// kernel of the stream has completed and its writes are visible; dep_launch()
+// lets the next kernel be scheduled.  Each such kernel keeps two rules:
+//  * a thread of every CTA returns from dep_wait() before the CTA reads what
+//    the previous kernel wrote, or writes memory that kernel reads or writes;
+//  * a CTA calls dep_launch() only in a thread that has returned from
+//    dep_wait().
+// So when a kernel is scheduled, every kernel before the previous one has
+// completed: what those wrote (the plan tables, the ranks behind the keep
+// lists) may be read before dep_wait().  Without the launch attribute both
+// instructions return at once.
+__device__ __forceinline__ void dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 }  // namespace vc

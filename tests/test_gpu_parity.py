@@ -398,3 +398,46 @@ def test_compress_per_layer_equals_step_api(kernel_path):
     torch.cuda.synchronize()
     assert torch.equal(idx, ref["keep"]) and torch.equal(Ko, ref["K_out"])
     assert torch.equal(Vo, ref["V_out"])
+
+
+def test_batch_with_tables_beyond_the_parameter_image(kernel_path):
+    """40 requests of 28 layers: every (request, layer) adds at least 36 bytes of
+    plan tables, so the image (> 40 KB) no longer travels as the upload kernel's
+    24 KB parameter; the call copies it with a memcpy and then clears the status
+    word with an upload of no bytes, and the kernels after it are ordered behind
+    that.  The batch equals every request compressed alone, bit for bit, and
+    three requests match the oracle."""
+    L, Hq, Hkv, d, nreq = 28, 8, 2, 128, 40
+    rng = np.random.default_rng(2608)
+    ns = [int(x) for x in rng.integers(200, 700, nreq)]
+    Ws = [int(x) for x in rng.integers(4, 17, nreq)]
+    rrs = [[(19, 100), (23, 100), (28, 100)][i % 3] for i in range(nreq)]
+    qs = [_rand((L, Hq, Ws[i], d), 7100 + 3 * i, torch.bfloat16) for i in range(nreq)]
+    ks = [_rand((L, Hkv, ns[i], d), 7101 + 3 * i, torch.bfloat16) for i in range(nreq)]
+    vs = [_rand((L, Hkv, ns[i], d), 7102 + 3 * i, torch.bfloat16) for i in range(nreq)]
+    Q = torch.cat([q.flatten() for q in qs]).to(DEV)
+    K = torch.cat([k.flatten() for k in ks]).to(DEV)
+    V = torch.cat([v.flatten() for v in vs]).to(DEV)
+    batch = vc.Batch(ns, Ws, rrs)
+    prm = vc.make_params(L, Hq, Hkv, d, vc.VC_BF16)
+    ws = torch.empty(vc.prunekv_workspace_size(batch, prm), dtype=torch.uint8, device=DEV)
+    ws.fill_(0xff)                       # a stale status word must be cleared by the call
+    Ko, Vo, idx = vc.prunekv_compress(batch, prm, Q, K, V, ws=ws)
+    assert vc.prunekv_get_status(ws) == vc.VC_OK
+    off = 0
+    for i in range(nreq):
+        one = vc.Batch([ns[i]], [Ws[i]], [rrs[i]])
+        rows = vc.compressed_rows(one, prm)
+        ko, vo, ix = vc.prunekv_compress(one, prm, qs[i].to(DEV), ks[i].to(DEV), vs[i].to(DEV))
+        torch.cuda.synchronize()
+        assert torch.equal(idx[off:off + rows], ix), "request %d idx" % i
+        assert torch.equal(Ko[off:off + rows], ko), "request %d K_out" % i
+        assert torch.equal(Vo[off:off + rows], vo), "request %d V_out" % i
+        if i in (0, nreq // 2, nreq - 1):
+            B, Nq, _ = vc.viscache_plan_budgets(L, ns[i], *rrs[i])
+            out = run_steps(qs[i].to(DEV), ks[i].to(DEV), vs[i].to(DEV), B, Nq)
+            assert torch.equal(out["keep"], ix) and torch.equal(out["K_out"], ko)
+            log = check_request(qs[i], ks[i], vs[i], B, Nq, out, 0.7, 1.0)
+            assert len(log) <= 2, log
+        off += rows
+    assert off == Ko.shape[0]

@@ -153,7 +153,13 @@ constexpr int kStages = 3;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSCol = 256;
 constexpr int kMaxUnits = 512;                   // units per pair (descriptor table)
-constexpr float kRescaleLog2 = 8.f;
+// The softmax keeps a row's reference maximum m until a tile's maximum
+// exceeds it by more than 2^32 (log2 units): until then P = 2^(x - m) stays
+// below 2^32, which bf16 P, the fp32 row sums and the fp32 O hold without
+// overflow, and only a larger rise rescales O.  Logits of 128-dimensional
+// rows spread over tens of log2 units, so a small threshold rescaled O on
+// most units' second tile.
+constexpr float kRescaleLog2 = 32.f;
 
 struct Unit {              // one unit as this CTA sees it
   int32_t vk_row;          // Vs row of this CTA's first kept row

@@ -441,3 +441,37 @@ def test_batch_with_tables_beyond_the_parameter_image(kernel_path):
             assert len(log) <= 2, log
         off += rows
     assert off == Ko.shape[0]
+
+
+@pytest.mark.parametrize("rise", [40.0, 300.0])
+def test_fusion_rescale_after_a_large_rise(rise):
+    """A dropped row in the fifth tile whose logit with kept row 5 exceeds that
+    row's maximum over the first four tiles by `rise` (log2 units, above the
+    fusion's 2^32 threshold) makes the softmax rescale the row's O and row sum;
+    without the rescale the earlier tiles' terms would outweigh it by 2^rise.
+    V_out of every kept row matches the oracle's fusion; K_out is exact."""
+    from oracle import prunekv as okp
+    from tests.parity import TOL, check_v_rows
+    L, Hkv, d, n, tau, mu = 1, 1, 128, 1200, 1.0, 0.3
+    B, Nq = [256], 1000                                   # 744 dropped rows: 6 tiles of 128
+    K = _rand((L, Hkv, n, d), 9101, torch.bfloat16)
+    V = _rand((L, Hkv, n, d), 9102, torch.bfloat16)
+    keep = np.arange(0, 256)
+    drop = np.arange(256, Nq)
+    r0, j_plant = 5, 256 + 4 * 128 + 17                   # kept row, planted token (tile 4)
+    v = V[0, 0].double().numpy()
+    m_prev = float((v[drop[:512]] @ v[r0]).max()) / tau * np.log2(np.e)
+    alpha = (m_prev + rise) * tau / (float(v[r0] @ v[r0]) * np.log2(np.e))
+    V[0, 0, j_plant] = (alpha * V[0, 0, r0].double()).to(torch.bfloat16)
+    v = V[0, 0].double().numpy()
+    got_rise = float(v[j_plant] @ v[r0]) / tau * np.log2(np.e) - m_prev
+    assert got_rise > 35.0, got_rise
+    ki = torch.tensor(keep, dtype=torch.int32, device=DEV)
+    di = torch.tensor(drop, dtype=torch.int32, device=DEV)
+    Ko, Vo = vc.prunekv_fuse_compact(K.to(DEV), V.to(DEV), B, Nq, ki, di, mu, tau)
+    torch.cuda.synchronize()
+    assert torch.equal(Ko.cpu(), K[0, 0][torch.from_numpy(keep)])
+    ref = okp.fuse_values(v, keep, drop, mu, tau)
+    check_v_rows(np64(Vo), ref, TOL[torch.bfloat16], "rise %g" % rise)
+    # the planted row dominates kept row 5's fused value
+    assert np.allclose(ref[r0], mu * v[r0] + (1 - mu) * v[j_plant], rtol=1e-6, atol=1e-6 * np.abs(v[j_plant]).max())

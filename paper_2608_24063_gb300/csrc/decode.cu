@@ -438,6 +438,75 @@ __device__ __forceinline__ void expand_q4(uint8_t* buf, const uint8_t* codes, co
   }
 }
 
+// 4-bit value rows staged in shared memory: the split's codes at byte 0
+// (D/2 bytes a row) and their parameters after kSplitM rows of codes (one
+// (scale, min) pair per row and 32-channel group).  Rows [0, kQ4StageRows)
+// of the row buffer hold them, so the staging is used when the split's text
+// rows (which load into rows nv ...) start at or after that row.
+template <int D>
+struct Q4Stage {
+  static constexpr int CODES = kSplitM * (D / 2);
+  static constexpr int BYTES = CODES + kSplitM * (D / 32) * 8;
+  static constexpr int ROWS = (BYTES + 2 * D - 1) / (2 * D);      // bf16 rows the staging covers
+  static_assert(BYTES <= (kSplitM / 2) * 2 * D, "the staging fits the first half of the row buffer");
+};
+
+// Copy the split's value codes and parameters into the staging area (16-byte
+// asynchronous copies; all addresses are 16-byte aligned).
+template <int D>
+__device__ __forceinline__ void stage_q4_values(uint32_t buf_s, const uint8_t* codes, const float* par, int nv) {
+  using S = Q4Stage<D>;
+  const uint8_t* pp = reinterpret_cast<const uint8_t*>(par);
+  const int nc = nv * (D / 2) / 16, np = nv * (D / 32) * 8 / 16;
+  for (int i = (int)threadIdx.x; i < nc + np; i += kDecThreads) {
+    const bool is_code = i < nc;
+    const uint32_t dst = buf_s + (is_code ? 16u * i : (uint32_t)S::CODES + 16u * (i - nc));
+    const uint8_t* src = is_code ? codes + 16 * i : pp + 16 * (i - nc);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+  }
+}
+
+// Value rows [0, nv) expanded from the staging area in two steps, so that no
+// thread overwrites codes another has not read: every thread first reads its
+// rows' codes and parameters (read_q4_values), then, after a barrier, writes
+// its bf16 rows (write_q4_values).  Thread t owns the 8-channel piece
+// t % PR of rows (t / PR) * RPT ..., as in expand_q4.
+template <int D>
+struct Q4Values {
+  static constexpr int RPT = kSplitM * (D / 8) / kDecThreads;   // as expand_q4: PR = D / 8 pieces a row
+  uint32_t w[RPT];
+  float2 p[RPT];
+};
+template <int D>
+__device__ __forceinline__ void read_q4_values(const uint8_t* buf, int nv, Q4Values<D>& v) {
+  using C = MmaCfg<D>;
+  constexpr int RPT = Q4Values<D>::RPT;
+  const int c = (int)threadIdx.x % C::PR, r0 = (int)threadIdx.x / C::PR * RPT;
+  const float2* par = reinterpret_cast<const float2*>(buf + Q4Stage<D>::CODES);
+#pragma unroll
+  for (int i = 0; i < RPT; ++i) {
+    const bool in = r0 + i < nv;
+    v.w[i] = in ? *reinterpret_cast<const uint32_t*>(buf + (size_t)(r0 + i) * (D / 2) + 4 * c) : 0u;
+    v.p[i] = in ? par[(size_t)(r0 + i) * (D / 32) + (c >> 2)] : make_float2(0.f, 0.f);
+  }
+}
+template <int D>
+__device__ __forceinline__ void write_q4_values(uint8_t* buf, int nv, const Q4Values<D>& v) {
+  using C = MmaCfg<D>;
+  constexpr int RPT = Q4Values<D>::RPT;
+  const int c = (int)threadIdx.x % C::PR, r0 = (int)threadIdx.x / C::PR * RPT;
+#pragma unroll
+  for (int i = 0; i < RPT; ++i) {
+    if (r0 + i >= nv) break;
+    float x[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) x[j] = fmaf((float)((v.w[i] >> (4 * j)) & 15u), v.p[i].x, v.p[i].y);
+    const int r = r0 + i;
+    *reinterpret_cast<uint4*>(buf + (size_t)r * C::RB + mma_slot(r, c) * 16) =
+        make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+  }
+}
+
 // Decode kernel for bf16 caches: one CTA per unit (request, KV head, split
 // of kSplitM keys), three CTAs per SM.  The split's K rows (with the query
 // rows) load first; its V rows load into the same buffer during the softmax.
@@ -478,6 +547,10 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   // [kHalf, 2 kHalf) during the softmax; PV takes the halves in turn.
   constexpr int kHalf = kSplitM / 2;
   static_assert(C::TPW == 2 && kHalf == 16 * kDecWarps, "QK tile h of every warp lies in half h");
+  // 4-bit: the value codes and parameters move into the first half of the row
+  // buffer while QK works on the second half (their load overlaps QK and the
+  // softmax), unless the split's text rows would land in the staging area
+  const bool q4_stage = Q4 && cur.nv >= Q4Stage<D>::ROWS;
   if (Q4) {
     stage_split<D>(buf_s, Kc, Kt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
     stage_q<D>(qbuf_s, q + ((int64_t)cur.r * tb.Hq + cur.g * G) * D, G);
@@ -520,6 +593,11 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   bool live[C::TPW];
 #pragma unroll
   for (int h = 0; h < C::TPW; ++h) {
+    if (q4_stage && h == 1) {
+      __syncthreads();                          // K rows [0, kHalf) read: stage the value codes there
+      stage_q4_values<D>(buf_s, Vq + cur.vis0 * (D / 2), Vqp + cur.vis0 * (D / 32) * 2, cur.nv);
+      tc::cp_async_commit();
+    }
     if (!Q4 && h == 1) {
       __syncthreads();                          // K rows [0, kHalf) read: V rows there
       stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q, 0, kHalf);
@@ -546,7 +624,7 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
   if (Q4) {
     stage_split<D>(buf_s, Vc, Vt + cur.txt0 * D, cur.nv, nk, q, cur.nv);
     tc::cp_async_commit();
-    expand_q4<D, false>(buf, Vq + cur.vis0 * (D / 2), Vqp + cur.vis0 * (D / 32) * 2, cur.nv);
+    if (!q4_stage) expand_q4<D, false>(buf, Vq + cur.vis0 * (D / 2), Vqp + cur.vis0 * (D / 32) * 2, cur.nv);
   } else {
     stage_split<D>(buf_s, Vc + cur.vis0 * D, Vt + cur.txt0 * D, cur.nv, nk, q, kHalf);
     tc::cp_async_commit();
@@ -602,9 +680,16 @@ __global__ void __launch_bounds__(kDecThreads, 3) decode_mma_kernel(
     wsum[warp * kGm + 2 * tig] = l0;
     wsum[warp * kGm + 2 * tig + 1] = l1;
   }
-  if (Q4) tc::cp_async_wait<0>();               // V rows
+  if (Q4) tc::cp_async_wait<0>();               // V rows (and the staged codes)
   else tc::cp_async_wait<1>();                  // V rows [0, kHalf)
   __syncthreads();
+  if (q4_stage) {
+    Q4Values<D> qv;
+    read_q4_values<D>(buf, cur.nv, qv);
+    __syncthreads();                            // every thread has its codes: overwrite them
+    write_q4_values<D>(buf, cur.nv, qv);
+    __syncthreads();
+  }
   if (t < G) {
     float M = wmax[t], L = 0.f;
 #pragma unroll

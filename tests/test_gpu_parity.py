@@ -475,3 +475,40 @@ def test_fusion_rescale_after_a_large_rise(rise):
     check_v_rows(np64(Vo), ref, TOL[torch.bfloat16], "rise %g" % rise)
     # the planted row dominates kept row 5's fused value
     assert np.allclose(ref[r0], mu * v[r0] + (1 - mu) * v[j_plant], rtol=1e-6, atol=1e-6 * np.abs(v[j_plant]).max())
+
+
+def test_concurrent_calls_on_two_streams():
+    """Calls on two streams with their own workspaces run at the same time (their
+    kernels are dependent launches within each stream, not across streams) and
+    give, bit for bit, what the same calls give one after the other; repeated
+    three times so the two streams' kernels interleave differently."""
+    wl = synth.scaled(synth.WORKLOADS[3], "7B shape, 8 layers, 4000 tokens", L=8,
+                      requests=[synth.Request(4000, 64, 19, 100, 100)])
+    wl2 = synth.scaled(synth.WORKLOADS[3], "7B shape, 8 layers, 2500 tokens", L=8,
+                       requests=[synth.Request(2500, 48, 28, 100, 101)])
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16)
+    inputs = []
+    for w in (wl, wl2):
+        q = synth.make_q(w, 0)
+        k, v = synth.make_kv(w, 0, q)
+        r = w.requests[0]
+        batch = vc.Batch([r.n], [r.W], [(r.rr_num, r.rr_den)])
+        inputs.append((batch, q.to(DEV), k.to(DEV), v.to(DEV)))
+    ref = []
+    for batch, Q, K, V in inputs:
+        ref.append(vc.prunekv_compress(batch, prm, Q, K, V))
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    wss = [torch.empty(vc.prunekv_workspace_size(b, prm), dtype=torch.uint8, device=DEV) for b, _, _, _ in inputs]
+    for rep in range(3):
+        outs = [None, None]
+        torch.cuda.synchronize()
+        for i in (0, 1) if rep % 2 == 0 else (1, 0):
+            batch, Q, K, V = inputs[i]
+            with torch.cuda.stream(streams[i]):
+                outs[i] = vc.prunekv_compress(batch, prm, Q, K, V, ws=wss[i], stream=streams[i])
+        torch.cuda.synchronize()
+        for i in (0, 1):
+            assert vc.prunekv_get_status(wss[i]) == vc.VC_OK
+            for a, b in zip(outs[i], ref[i]):
+                assert torch.equal(a, b), "rep %d stream %d" % (rep, i)

@@ -61,7 +61,7 @@ extern "C" {
 #define VC_ERR_WORKSPACE        3  /* workspace NULL, misaligned or smaller than required */
 #define VC_ERR_CUDA             4  /* a CUDA runtime call or kernel launch failed */
 #define VC_ERR_DEVICE_TIMEOUT   5  /* a bounded device-side wait gave up */
-#define VC_ERR_UNSUPPORTED      6  /* valid request outside what this build implements */
+#define VC_ERR_UNSUPPORTED      6  /* valid request outside what the library implements */
 #define VC_ERR_DEVICE_INDEX     7  /* a kernel met an index out of range and skipped it */
 
 /* ---- element types ---- */

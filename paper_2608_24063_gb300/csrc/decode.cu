@@ -16,8 +16,11 @@
 //                          finishes the last split of a (request, KV head)
 //                          merges the pair's split states into the output.
 //                          Its Q4 form reads the visual rows from the 4-bit
-//                          cache (codes and parameters loaded into registers
-//                          and expanded to bf16 rows in the same buffer).
+//                          cache: key codes and parameters loaded into
+//                          registers and expanded to bf16 rows in the same
+//                          buffer; value codes and parameters copied into
+//                          shared memory during QK and expanded after the
+//                          softmax.
 //   decode_partial_kernel  (fp32 caches, splits of 256 keys) the same steps on
 //                          CUDA cores, K then V rows in one buffer: two
 //                          threads per key pair form the logits with packed

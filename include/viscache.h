@@ -449,6 +449,19 @@ int viscache_kv4_dequantize(const vc_batch* batch, const vc_params* p, const uin
 int viscache_set_kernel_path(int path);
 
 /*
+ * Launch ordering (process-wide, default 1): with 1 the kernels of a call
+ * after its first are programmatic dependent launches -- each may be
+ * scheduled while the kernel before it on the stream drains, and waits on
+ * the device for that kernel's results before it reads them -- which hides
+ * the gaps between them; with 0 every kernel is an ordinary launch and starts
+ * only when the previous one has completed.  Results are the same either
+ * way; 0 is for debugging and for timing the difference.  Calls are never
+ * overlapped with work queued before them: a call's first kernel is always
+ * an ordinary launch.  Errors: VC_ERR_INVALID_ARG unless on is 0 or 1.
+ */
+int viscache_set_dependent_launch(int on);
+
+/*
  * viscache_test_inject_wait -- test support for the failure detection of the
  * tensor-core kernels (not a step of the pass).  For every later launch of
  * a kernel named in kernel_mask, one consumer warp first waits on an

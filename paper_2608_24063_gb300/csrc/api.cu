@@ -14,6 +14,15 @@
 #include "vc_common.cuh"
 
 namespace vc {
+
+// Programmatic dependent launches between the kernels of a call (launch_dep);
+// 0 launches every kernel fully serialised.
+#ifdef VC_SERIAL_LAUNCH
+std::atomic<int> g_dependent_launch{0};
+#else
+std::atomic<int> g_dependent_launch{1};
+#endif
+
 namespace {
 
 constexpr size_t kAlign = 256;
@@ -577,6 +586,12 @@ int viscache_test_inject_wait(int kernel_mask) {
   if (kernel_mask < 0 || kernel_mask > (VC_TEST_WAIT_SCORE_LSE | VC_TEST_WAIT_SCORE_COLSUM | VC_TEST_WAIT_FUSE))
     return VC_ERR_INVALID_ARG;
   g_test_wait.store(kernel_mask);
+  return VC_OK;
+}
+
+int viscache_set_dependent_launch(int on) {
+  if (on != 0 && on != 1) return VC_ERR_INVALID_ARG;
+  vc::g_dependent_launch.store(on);
   return VC_OK;
 }
 

@@ -3,14 +3,20 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "vc_common.cuh"
 
 namespace vc {
 
+// 1 (default): launch_dep lets a kernel start while the one before it drains;
+// 0 (viscache_set_dependent_launch, or built with VC_SERIAL_LAUNCH): every
+// kernel waits for the previous one to complete, as an ordinary launch.
+extern std::atomic<int> g_dependent_launch;
+
 // Launches kernel on st so that it may be scheduled before the previous kernel
 // on the stream has completed (programmatic stream serialisation); the kernel
-// orders itself with dep_wait / dep_launch (vc_common.cuh).  Defining
-// VC_SERIAL_LAUNCH launches every kernel fully serialised instead.
+// orders itself with dep_wait / dep_launch (vc_common.cuh).
 template <typename... P, typename... A>
 cudaError_t launch_dep(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                        A&&... args) {
@@ -23,11 +29,7 @@ cudaError_t launch_dep(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem,
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cfg.attrs = at;
-#ifdef VC_SERIAL_LAUNCH
-  cfg.numAttrs = 0;
-#else
-  cfg.numAttrs = 1;
-#endif
+  cfg.numAttrs = g_dependent_launch.load(std::memory_order_relaxed) ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<A&&>(args)...);
 }
 

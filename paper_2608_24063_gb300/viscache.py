@@ -40,7 +40,8 @@ EXPORTED = ("viscache_plan_budgets", "viscache_plan_budgets_ex", "prunekv_score_
             "prunekv_fuse_compact", "prunekv_workspace_size", "prunekv_compress",
             "prunekv_get_status", "viscache_version", "viscache_profile_enable",
             "viscache_profile_read", "prunekv_score_static", "prunekv_score_static_capacity",
-            "prunekv_score_static_status", "viscache_set_kernel_path", "viscache_test_inject_wait",
+            "prunekv_score_static_status", "viscache_set_kernel_path", "viscache_set_dependent_launch",
+            "viscache_test_inject_wait",
             "viscache_device_accessible", "viscache_scout_workspace_size", "viscache_scout_sizes", "viscache_scout_mmr",
             "viscache_decode_workspace_size", "viscache_decode_attention",
             "viscache_kv4_sizes", "viscache_kv4_quantize", "viscache_kv4_dequantize",
@@ -122,6 +123,7 @@ def lib() -> ctypes.CDLL:
         L.viscache_version.restype = ctypes.c_char_p
         L.viscache_profile_enable.argtypes = [i32]
         L.viscache_set_kernel_path.argtypes = [i32]
+        L.viscache_set_dependent_launch.argtypes = [i32]
         L.viscache_test_inject_wait.argtypes = [i32]
         L.viscache_device_accessible.argtypes = [vp]
         L.viscache_profile_read.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(ctypes.c_float),
@@ -485,6 +487,11 @@ def viscache_kv4_dequantize(batch: Batch, params: vc_params, K_codes: torch.Tens
 def viscache_set_kernel_path(path: int) -> None:
     """VC_PATH_AUTO (tensor cores for bf16, d=128) or VC_PATH_SIMT (CUDA cores everywhere)."""
     _check("viscache_set_kernel_path", lib().viscache_set_kernel_path(path))
+
+
+def viscache_set_dependent_launch(on: bool) -> None:
+    """True (default): kernels after a call's first are dependent launches; False: ordinary launches."""
+    _check("viscache_set_dependent_launch", lib().viscache_set_dependent_launch(1 if on else 0))
 
 
 def viscache_test_inject_wait(kernel_mask: int) -> None:

@@ -512,3 +512,35 @@ def test_concurrent_calls_on_two_streams():
             assert vc.prunekv_get_status(wss[i]) == vc.VC_OK
             for a, b in zip(outs[i], ref[i]):
                 assert torch.equal(a, b), "rep %d stream %d" % (rep, i)
+
+
+@pytest.fixture
+def dependent_launch():
+    yield vc.viscache_set_dependent_launch
+    vc.viscache_set_dependent_launch(True)
+
+
+@pytest.mark.parametrize("wid", [3, 5])
+def test_dependent_launches_give_the_same_bits(wid, dependent_launch):
+    """The whole pass (and the step API) with the kernels of a call launched as
+    dependent launches and as ordinary launches: equal bit for bit (workload 3,
+    the 7B shape at 12,544 tokens, and the ragged 8-request batch)."""
+    wl = synth.WORKLOADS[wid]
+    qs, ks, vs = synth.generate(wl, DEV)
+    Q = torch.cat([q.flatten() for q in qs])
+    K = torch.cat([k.flatten() for k in ks])
+    V = torch.cat([v.flatten() for v in vs])
+    batch = vc.Batch([r.n for r in wl.requests], [r.W for r in wl.requests],
+                     [(r.rr_num, r.rr_den) for r in wl.requests])
+    prm = vc.make_params(wl.L, wl.Hq, wl.Hkv, wl.d, vc.VC_BF16)
+    outs = {}
+    for on in (True, False, True):
+        dependent_launch(on)
+        res = vc.prunekv_compress(batch, prm, Q, K, V)
+        s = vc.prunekv_score(qs[0], ks[0])
+        torch.cuda.synchronize()
+        outs.setdefault(on, []).append(tuple(t.clone() for t in res) + (s.clone(),))
+    ref = outs[True][0]
+    for got in outs[True][1:] + outs[False]:
+        for a, b in zip(got, ref):
+            assert torch.equal(a, b)
